@@ -1,0 +1,418 @@
+#!/usr/bin/env python
+"""Benchmark: batch-1 FP32 decode tokens/s of the 110M Llama-2-shape model.
+
+A step is one decode step (all layers + classifier + greedy argmax) for one
+token. The timed region runs K steps as greedy sequences of 256 steps from
+token 1 (the paper's 256-token run), each sequence one launch of the
+persistent decode kernel, with the weights resident in HBM. Weights streamed
+per step (438 MB) exceed L2 (~126 MB), so no L2 flush is needed between steps.
+
+Printed JSON line (rank 0): value = tokens/s over all ranks; e2e = the same
+metric through tvl_forward with host logits (token in, 128 KB of logits out,
+host argmax, every step); roofline of the decode kernel against the measured
+HBM copy bandwidth; cpu_baseline = the CPU oracle on the host cores.
+
+--impl reference times the CPU oracle (the only reference this paper has; it
+publishes no code) on the same workload.
+
+Multi-GPU (torchrun): replicas only — each rank decodes its own sequences; no
+collective on the data path. value = all ranks' tokens / max rank time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "batch-1 decode tokens/s (110M FP32); GEMV HBM GB/s vs ~8 TB/s peak"
+PAPER_TOKS = 61.3  # the paper's 110M FP32 decode on one M2 Pro core (Table 1)
+SEQ = 256
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=4096)
+    ap.add_argument("--warmup", type=int, default=256)
+    ap.add_argument("--impl", default="tvl", choices=["tvl", "reference"])
+    ap.add_argument("--workload", default="110m", choices=["110m", "tiny", "7b"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--gemv-sweep", action="store_true", help="GEMV GB/s per shape instead")
+    return ap.parse_args()
+
+
+def dist_env():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)),
+            int(os.environ.get("WORLD_SIZE", 1)))
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2601_03324_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(f.encode() + fh.read())
+    return h.hexdigest()[:16]
+
+
+def committed_traffic(workload: str):
+    """dram bytes per step from the committed ncu summary, if it was taken
+    on the kernel sources as they are now."""
+    p = os.path.join(ROOT, "profiles", f"decode_kernel_{workload}.txt")
+    if not os.path.exists(p):
+        return None
+    kv = {}
+    for line in open(p):
+        if ":" in line:
+            k, v = line.split(":", 1)
+            kv[k.strip()] = v.strip()
+    if kv.get("kernel_sources_sha256_16") != kernel_hash():
+        return None
+    try:
+        return float(kv["dram_bytes_per_step"])
+    except (KeyError, ValueError):
+        return None
+
+
+def step_bytes(cfg: dict, streamed: int, pos: int) -> int:
+    """Algorithmic bytes of one step at position pos: every weight once, the
+    K/V cache rows of positions < pos, the new K/V row, the logits."""
+    d, L, V = cfg["dim"], cfg["n_layers"], cfg["vocab_size"]
+    kvd = cfg["n_kv_heads"] * (d // cfg["n_heads"])
+    return streamed + 2 * pos * kvd * 4 * L + 2 * kvd * 4 * L + 4 * V
+
+
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, dev_index: int, uuid: str | None):
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+        os.makedirs(os.path.dirname(self.path), exist_ok=True)
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+               "-lms", "50"]
+        cmd += ["-i", uuid] if uuid else ["-i", str(dev_index)]
+        try:
+            self.f = open(self.path, "w")
+            self.p = subprocess.Popen(cmd, stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.p = None
+
+    def stop(self, t0: float, t1: float):
+        if self.p is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.12)
+        self.p.terminate()
+        try:
+            self.p.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.p.kill()
+        self.f.close()
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                ts = time.mktime(time.strptime(parts[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                ts += float("0." + parts[0].split(".")[1]) if "." in parts[0] else 0.0
+                rows.append((ts, float(parts[1]), float(parts[2]), parts[5:9]))
+            except (ValueError, IndexError):
+                continue
+        win = [r for r in rows if t0 - 0.06 <= r[0] <= t1 + 0.06] or rows[-3:]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in win for i, v in enumerate(r[3]) if v == "Active"})
+        return {"sm_mhz": statistics.median([r[1] for r in win]) if win else None,
+                "sm_max_mhz": max(r[2] for r in win) if win else None,
+                "reasons": reasons, "samples": len(win)}
+
+
+def cpu_oracle_rate(cfg, blob, seconds: float):
+    """The CPU oracle (double accumulators, one thread) decoding greedily from
+    token 1 for about `seconds`; tokens/s."""
+    import oracle
+    m = oracle.Model(cfg, blob, 64)
+    t, n = 1, 0
+    t0 = time.perf_counter()
+    while True:
+        lg = m.forward(t, n)
+        t = int(np.argmax(lg))
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= seconds or n >= cfg["max_seq"]:
+            break
+    return n / el, n, el
+
+
+def run_reference(args, cfg, rank, world):
+    if rank != 0:
+        return 0
+    from paper_2601_03324_gb300 import synth
+    import oracle
+    blob = synth.make_blob(cfg)
+    m = oracle.Model(cfg, blob, 64)
+    t = 1
+    for s in range(args.warmup):
+        t = int(np.argmax(m.forward(t, s % cfg["max_seq"])))
+    # size each step so the whole run stays within ~150 s: a whole token when
+    # that fits, else the same fraction of every weight matrix's rows
+    t0 = time.perf_counter()
+    m.forward(t, 0)
+    t_tok = time.perf_counter() - t0
+    frac = min(1.0, 150.0 / max(1e-9, args.steps * t_tok))
+    t0 = time.perf_counter()
+    if frac >= 1.0:
+        pos = 0
+        for s in range(args.steps):
+            t = int(np.argmax(m.forward(t, pos)))
+            pos = (pos + 1) % SEQ
+            if pos == 0:
+                t = 1
+        sample = f"{args.steps} whole decode steps of the workload (greedy, 256-step sequences)"
+    else:
+        from paper_2601_03324_gb300 import synth as sy
+        mats = [(n, l) for l in range(cfg["n_layers"])
+                for n in ("Wq", "Wk", "Wv", "Wo", "W1", "W3", "W2")] + [("Wcls", -1)]
+        xs = {}
+        for s in range(args.steps):
+            for (n, l) in mats:
+                W = sy.tensor(blob, cfg, n, l)
+                rows = max(1, int(math.ceil(frac * W.shape[0])))
+                if W.shape[1] not in xs:
+                    xs[W.shape[1]] = np.ones(W.shape[1])
+                oracle.gemv(W[:rows], xs[W.shape[1]])
+        sample = (f"each step: the oracle GEMV over {frac:.4f} of every weight matrix's rows "
+                  f"(the GEMVs are the step's cost), scaled to whole steps")
+    el = time.perf_counter() - t0
+    val = args.steps * frac / el
+    line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "tokens/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000.0 * el / (args.steps * frac), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": val / PAPER_TOKS, "dtype": "f64",
+            "data": "synthetic", "config": workload_config(args.workload, cfg),
+            "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config(name, cfg):
+    desc = {"110m": "110M Llama-2-shape FP32 decoder (d768 L12 H12 F2048 V32000, tied), "
+                    "batch 1, greedy 256-step sequences from token 1",
+            "tiny": "tiny Llama-2-shape FP32 decoder (d288 L6 H6 F768 V32000), batch 1",
+            "7b": "7B Llama-2-shape FP32 decoder (d4096 L32 H32 F11008 V32000), batch 1, "
+                  "greedy 16-step sequences"}[name]
+    return {"workload": desc, "seq_steps": min(SEQ, cfg["max_seq"]), "batch": 1,
+            "weights_seed": cfg["seed"], "parallelism": "replicas",
+            "l2": "inputs larger than L2: every step streams all weights (> L2 size)"}
+
+
+def gemv_sweep(args):
+    import torch
+    from paper_2601_03324_gb300 import synth, tvl
+    torch.cuda.set_device(0)
+    l2 = torch.cuda.get_device_properties(0).L2_cache_size
+    s = torch.cuda.Stream()
+    out = []
+    for i, (M, K) in enumerate(synth.GEMV_SHAPES):
+        W, x = synth.gemv_operands(M, K, i)
+        nbytes = 4 * (M * K + M + K)
+        copies = max(1, math.ceil(3 * l2 / (4 * M * K)))
+        dW = torch.from_numpy(W).cuda().repeat(copies, 1).reshape(copies, M, K)
+        dx = torch.from_numpy(x).cuda()
+        dy = torch.empty(M, device="cuda")
+        reps = 200
+        with torch.cuda.stream(s):
+            for r in range(10):
+                tvl.tvl_gemv(dW[r % copies].data_ptr(), dx.data_ptr(), dy.data_ptr(), M, K,
+                             s.cuda_stream)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=s):
+                for r in range(reps):
+                    tvl.tvl_gemv(dW[r % copies].data_ptr(), dx.data_ptr(), dy.data_ptr(), M, K,
+                                 s.cuda_stream)
+            g.replay()
+            s.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(s)
+            g.replay()
+            e1.record(s)
+        e1.synchronize()
+        us = e0.elapsed_time(e1) * 1000.0 / reps
+        out.append({"shape": [M, K], "us": us, "GB/s": nbytes / us / 1e3, "cold_copies": copies})
+        del dW, g
+    peak, src = measured_peaks()
+    for o in out:
+        o["frac_of_" + src + "_hbm"] = o["GB/s"] / peak
+    print(json.dumps({"gemv_sweep": out, "peak_gbs": peak, "peak_source": src}), flush=True)
+
+
+def main():
+    args = parse()
+    rank, local_rank, world = dist_env()
+    from paper_2601_03324_gb300 import synth
+    cfg = synth.model_config(args.workload)
+    if args.impl == "reference":
+        return run_reference(args, cfg, rank, world)
+    import torch
+    import torch.distributed as dist
+    if args.gemv_sweep:
+        return gemv_sweep(args)
+    if world > 1:
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local_rank)
+    from paper_2601_03324_gb300 import tvl
+
+    blob = synth.make_blob(cfg)
+    stream = torch.cuda.Stream()
+    model = tvl.Model(cfg, blob, stream=stream.cuda_stream)
+    info = model.info()
+    seq = min(SEQ, cfg["max_seq"])
+
+    def run_steps(k, events=None):
+        """k decode steps as greedy sequences of `seq` steps (one launch each)."""
+        launches = 0
+        done = 0
+        while done < k:
+            n = min(seq, k - done)
+            if events is not None:
+                e0 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+            model.decode_greedy(1, 0, n, tokens=False)
+            if events is not None:
+                e1 = torch.cuda.Event(enable_timing=True)
+                e1.record(stream)
+                events.append((e0, e1, n))
+            done += n
+            launches += 1
+        return launches
+
+    run_steps(max(3, args.warmup))
+    model.sync()
+    props = torch.cuda.get_device_properties(local_rank)
+    uuid = getattr(props, "uuid", None)
+    uuid = f"GPU-{uuid}" if uuid and not str(uuid).startswith("GPU-") else (str(uuid) if uuid else None)
+    clocks = Clocks(local_rank, uuid)
+    time.sleep(0.15)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ev = []
+    t_wall0 = time.time()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    launches = run_steps(args.steps, ev)
+    end.record(stream)
+    model.sync()
+    torch.cuda.synchronize()
+    t_wall1 = time.time()
+    if world > 1:
+        dist.barrier()
+    el_ms = start.elapsed_time(end)
+    clk = clocks.stop(t_wall0, t_wall1)
+    el_t = torch.tensor([el_ms], device="cuda")
+    if world > 1:
+        dist.all_reduce(el_t, op=dist.ReduceOp.MAX)
+    el_ms = float(el_t.item())
+
+    # per-launch roofline of the decode kernel (full-length launches)
+    full = [(a.elapsed_time(b), n) for (a, b, n) in ev]
+    launch_ms = statistics.mean(t for t, n in full)
+    n_typ = full[0][1]
+    bytes_launch = sum(step_bytes(cfg, info.streamed_bytes, p) for p in range(n_typ))
+    peak, peak_src = measured_peaks()
+    achieved = bytes_launch / (statistics.mean(t for t, n in full if n == n_typ) * 1e-3) / 1e9
+    traffic = committed_traffic(args.workload)
+    steps_ns = model.step_times(n_typ).astype(np.float64)
+    dts = np.diff(steps_ns) / 1e3 if n_typ > 1 else np.array([launch_ms * 1e3])
+
+    # end to end through the public API: token in, host logits out, host argmax
+    e2e = None
+    if not args.no_e2e:
+        import torch as _t
+        host_logits = _t.empty(cfg["vocab_size"], dtype=_t.float32, pin_memory=True).numpy()
+        k_e2e = min(args.steps, 2048)
+        tok = 1
+        for p in range(8):
+            model.forward(tok, p, host_logits)
+            tok = int(np.argmax(host_logits))
+        t0 = time.perf_counter()
+        tok, pos = 1, 0
+        for s in range(k_e2e):
+            model.forward(tok, pos, host_logits)
+            tok = int(np.argmax(host_logits))
+            pos += 1
+            if pos == seq:
+                tok, pos = 1, 0
+        e2e_s = time.perf_counter() - t0
+        e2e = {"value": world * k_e2e / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": 4,
+               "d2h_bytes_per_step": 4 * cfg["vocab_size"],
+               "note": "tvl_forward per step: token as launch argument, logits to pinned host "
+                       "memory, argmax on the host"}
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline and args.workload != "7b":
+        rate, n, el = cpu_oracle_rate(cfg, blob, args.cpu_seconds)
+        cpu = {"value": rate, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+               "sample": f"first {n} greedy steps of the workload from token 1 "
+                         f"({el:.1f} s, double accumulators, one thread)"}
+
+    value = world * args.steps / (el_ms * 1e-3)
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": el_ms / args.steps,
+        "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": value / PAPER_TOKS if args.workload == "110m" else None,
+        "dtype": "f32", "data": "synthetic (seeded N(0, 0.02) weights)",
+        "config": workload_config(args.workload, cfg),
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "kernel": "decode_kernel", "peak_source": peak_src,
+                     "bytes_per_launch": bytes_launch, "steps_per_launch": n_typ,
+                     "launch_ms": launch_ms},
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": launches,
+        "clocks": clk,
+        "step_latency_us": {"p50": float(np.percentile(dts, 50)),
+                            "p99": float(np.percentile(dts, 99))},
+        "grid": info.grid, "ring_stages": info.ring_stages,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    model.close()
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main() or 0)

@@ -1,0 +1,159 @@
+/*
+ * tvl.h — C ABI of the GB300 batch-1 FP32 decode library (libtvl.so).
+ *
+ * The library runs the single-token decode step of a Llama-2-architecture
+ * decoder on one GPU (sm_103a): every weight is streamed from HBM once per
+ * token through y = W x products, as the paper frames the problem
+ * (Kilictas & Alpay, "Bare-Metal Tensor Virtualization", arXiv 2601.03324,
+ * §1 and §3.1). The weights live in one device arena filled by a single
+ * host-to-device copy of a packed blob (§4.1, mmap'd model file; §3.2,
+ * aligned buffers).
+ *
+ * Conventions for every entry point:
+ *   - No exception crosses the ABI; every call returns a tvl_status.
+ *     tvl_last_error() gives a message for the calling thread's last failure.
+ *   - A tvl_model handle is not thread-safe: one host thread at a time.
+ *   - "stream" arguments are cudaStream_t values passed as void*.
+ *   - All tensors are float32; matrices are row-major [rows x cols].
+ */
+#ifndef TVL_H
+#define TVL_H
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  TVL_OK = 0,
+  TVL_E_INVAL = 1,       /* bad argument or configuration */
+  TVL_E_SIZE = 2,        /* blob size differs from tvl_blob_bytes() */
+  TVL_E_ALIGN = 3,       /* pointer alignment the kernel needs is missing */
+  TVL_E_NOMEM = 4,       /* device or pinned host allocation failed */
+  TVL_E_CUDA = 5,        /* a CUDA runtime call failed (see tvl_last_error) */
+  TVL_E_RANGE = 6,       /* token, position or step count out of range */
+  TVL_E_TIMEOUT = 7,     /* a bounded device-side wait gave up; model unusable */
+  TVL_E_UNSUPPORTED = 8  /* shape the GPU path does not handle (see tvl_load) */
+} tvl_status;
+
+/* Model shape. Paper §2.1: RMSNorm pre-normalisation, SwiGLU FFN with three
+ * matrices, RoPE on q and k; §5.1: classifier tied to the token embedding. */
+typedef struct {
+  int32_t dim;          /* d, model width */
+  int32_t hidden_dim;   /* F, SwiGLU hidden width */
+  int32_t n_layers;     /* L (0 allowed: embedding -> final norm -> classifier) */
+  int32_t n_heads;      /* H query heads; head_dim = d / H */
+  int32_t n_kv_heads;   /* Hkv key/value heads; H % Hkv == 0 (query head h uses h / (H/Hkv)) */
+  int32_t vocab_size;   /* V */
+  int32_t max_seq;      /* S, KV-cache positions */
+  double rope_theta;    /* RoPE base (10000) */
+  double norm_eps;      /* RMSNorm epsilon, added to mean(x^2) inside the sqrt (1e-5, §11.2) */
+  int32_t shared_classifier; /* 1 tied (Wcls is E), 0 untied, -1 infer from blob size (§5.1) */
+} tvl_config;
+
+typedef struct tvl_model tvl_model; /* opaque: device arena, stream, kernel plan */
+
+/* Exact byte size of the packed blob for cfg, tied (1) or untied (0)
+ * classifier; 0 if cfg is invalid.
+ * Blob layout (the paper's "Tensor Virtualization Layout", §4.1, which it
+ * leaves undefined; this is the definition used here): float32 row-major
+ * tensors, each starting at a 128-byte-aligned offset (zero padding), in the
+ * order  E[V x d];  per layer  g_att[d], Wq[d x d], Wk[kvd x d], Wv[kvd x d],
+ * Wo[d x d], g_ffn[d], W1[F x d], W3[F x d], W2[d x F];  g_final[d];
+ * Wcls[V x d] unless tied.  (kvd = Hkv * d / H.) */
+size_t tvl_blob_bytes(const tvl_config* cfg, int32_t tied);
+
+/* Load a model: pins `blob` (host memory owned by the caller, typically an
+ * mmap of the model file, §4.1) if it is not pinned already, copies it with
+ * ONE host-to-device transfer into a 256-byte-aligned device arena, builds
+ * the RoPE table and zeroes the KV cache. On return the caller may free or
+ * unmap `blob`.
+ *   cfg        model shape; shared_classifier -1 takes the paper's heuristic
+ *              (a blob one classifier short is tied).
+ *   blob_bytes must equal tvl_blob_bytes(cfg, tied), else TVL_E_SIZE.
+ *   stream     cudaStream_t for all work on this model; NULL: the library
+ *              creates and owns a non-blocking stream.
+ *   out        receives the handle (NULL on failure).
+ * GPU-path requirements (else TVL_E_UNSUPPORTED): dim % 32 == 0,
+ * head_dim % 4 == 0 and <= 256, hidden_dim % 4 == 0, max(dim, hidden_dim)
+ * <= 16384. Invalid shapes give TVL_E_INVAL. Uses the current CUDA device. */
+tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, void* stream,
+                    tvl_model** out);
+
+/* Same, from a file: mmap(PROT_READ, MAP_PRIVATE | MAP_POPULATE) of `path`
+ * (§4.1, and the Linux pre-fault hint of the artifact appendix), then
+ * tvl_load on the mapping, then munmap. */
+tvl_status tvl_load_file(const tvl_config* cfg, const char* path, void* stream, tvl_model** out);
+
+/* One decode step (§7.1: the timed unit is one forward() call returning the
+ * logits): embeds `token` at position `pos`, runs every layer (writing K/V
+ * of this position into the cache) and the classifier.
+ *   0 <= token < V and 0 <= pos < max_seq, else TVL_E_RANGE. Positions
+ *   0..pos-1 must hold this sequence's K/V (call positions in order;
+ *   calling a position again overwrites it).
+ *   logits_out: V floats. Device pointer: the copy is queued on the model
+ *   stream and the call returns without waiting. Host pointer: the call waits
+ *   and then reports device-side errors. NULL: logits stay on the device.
+ * The whole step is one kernel launch (a persistent kernel). */
+tvl_status tvl_forward(tvl_model* m, int32_t token, int32_t pos, float* logits_out);
+
+/* Greedy decoding kept on the device (§9.1 names greedy decoding as the
+ * baseline strategy; §7.1 generates 256 tokens): n_steps decode steps in ONE
+ * kernel launch, starting with start_token at start_pos; the token fed at each
+ * later step is the argmax of the previous logits (lowest index on ties).
+ *   tokens_out: host array of n_steps; tokens_out[s] = argmax after step s.
+ *   NULL: nothing is copied and the call does not wait.
+ *   start_pos + n_steps <= max_seq, n_steps >= 1, else TVL_E_RANGE. */
+tvl_status tvl_decode_greedy(tvl_model* m, int32_t start_token, int32_t start_pos,
+                             int32_t n_steps, int32_t* tokens_out);
+
+/* Standalone GEMV y = W x (§6.1), W [d_out x d_in] row-major, x [d_in],
+ * y [d_out]; all device pointers; queued on `stream` (NULL = default stream),
+ * does not wait. d_out >= 1, d_in >= 1, else TVL_E_INVAL. The fast path
+ * (TMA bulk staging) needs W and x 16-byte aligned and d_in % 4 == 0 and
+ * d_in <= 16384; other shapes take a plain per-row kernel. Deterministic: the
+ * same inputs give the same bits. A per-stream scratch buffer (a few KB) is
+ * allocated on first use for short-and-wide shapes and kept until exit;
+ * concurrent calls on different streams are safe. */
+tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t d_out, int32_t d_in,
+                    void* stream);
+
+/* Wait for the model's queued work, then report any device-side error. */
+tvl_status tvl_sync(tvl_model* m);
+
+/* Release the device arena and the stream the library created. NULL is ignored. */
+void tvl_free(tvl_model* m);
+
+const char* tvl_status_string(tvl_status s);
+const char* tvl_last_error(void);
+
+/* Facts about a loaded model, for benchmarks and tests. */
+typedef struct {
+  int64_t arena_bytes;       /* the single device allocation */
+  int64_t weight_bytes;      /* the blob as copied */
+  int64_t streamed_bytes;    /* weight bytes read per decode step */
+  int32_t grid;              /* persistent CTAs (one per SM) */
+  int32_t threads;           /* threads per CTA */
+  int32_t smem_bytes;        /* dynamic shared memory per CTA */
+  int32_t ring_stages;       /* weight staging ring: stages x stage_bytes */
+  int32_t stage_bytes;
+  int32_t tied;
+  int32_t barriers_per_step; /* grid-wide barriers in one greedy step */
+} tvl_model_info;
+tvl_status tvl_get_info(const tvl_model* m, tvl_model_info* out);
+
+/* Device timestamps (ns, %globaltimer) taken at the end of each step of the
+ * last tvl_decode_greedy call, for per-step latency statistics (§7.3). */
+tvl_status tvl_step_times(tvl_model* m, uint64_t* ns_out, int32_t n);
+
+/* Failure-detection self-test: launches the grid barrier of the decode kernel
+ * against a count that nothing will reach, with a wait limit of limit_ms.
+ * Expected result TVL_E_TIMEOUT, reported by the kernel itself, with the CUDA
+ * context still usable. Uses the current device. */
+tvl_status tvl_selftest_barrier_timeout(int32_t limit_ms);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* TVL_H */

@@ -1,0 +1,493 @@
+// decode.cu — model loading (one host-to-device copy into one arena) and the
+// launches of the persistent decode kernel, behind the C ABI of include/tvl.h.
+#include <fcntl.h>
+#include <sys/mman.h>
+#include <sys/stat.h>
+#include <unistd.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "decode_kernel.cuh"
+#include "host_common.h"
+
+using namespace tvl;
+
+struct tvl_model {
+  tvl_config cfg{};
+  bool tied = false;
+  int device = 0;
+  cudaStream_t stream = nullptr;
+  bool own_stream = false;
+  unsigned char* arena = nullptr;
+  size_t arena_bytes = 0;
+  size_t weight_bytes = 0;
+  int64_t streamed_bytes = 0;
+  DecodeArgs args{};
+  int smem_bytes = 0;
+  int* err_host = nullptr;  // pinned, mapped: the kernel writes its error code here too
+  tvl_status sticky = TVL_OK;
+};
+
+namespace {
+
+struct SmemPlan {
+  int ring, bars, xs, vec, pdot, att, misc, total, nst;
+};
+
+SmemPlan plan_smem(int d, int F, int hd, int H, int nch_cap, int max_bytes) {
+  SmemPlan p{};
+  const int att_floats =
+      std::max(3 * hd + kAttMaxChunk + 4 * kConsumerThreads, 2 * H * nch_cap) + 16;
+  const int xs = (int)a128(4LL * d), vec = (int)a128(4LL * std::max(d, F));
+  const int pdot = 2 * kMaxPieces * 4, att = (int)a128(4LL * att_floats), misc = 256;
+  const int bars = 2 * 8 * 8;
+  const int other = bars + xs + vec + pdot + att + misc;
+  int nst = (max_bytes - other) / kStageBytes;
+  if (nst > 8) nst = 8;
+  p.nst = nst;
+  int off = 0;
+  p.ring = off;
+  off += nst * kStageBytes;
+  p.bars = off;
+  off += bars;
+  p.xs = off;
+  off += xs;
+  p.vec = off;
+  off += vec;
+  p.pdot = off;
+  off += pdot;
+  p.att = off;
+  off += att;
+  p.misc = off;
+  off += misc;
+  p.total = off;
+  return p;
+}
+
+int nch_cap_for(int S, int H, int G) {
+  int cap = 1;
+  for (int pos = 0; pos < S; ++pos) {
+    int nch, clen;
+    att_split(pos, H, G, &nch, &clen);
+    cap = std::max(cap, nch);
+  }
+  return cap;
+}
+
+tvl_status check_device_error(tvl_model* m) {
+  const int code = *reinterpret_cast<volatile int*>(m->err_host);
+  if (code != 0) {
+    m->sticky = (tvl_status)code;
+    set_error("a bounded device-side wait expired (grid barrier or stage copy); "
+              "the model's device state is no longer consistent");
+    return m->sticky;
+  }
+  return TVL_OK;
+}
+
+void destroy(tvl_model* m) {
+  if (!m) return;
+  if (m->arena) cudaFree(m->arena);
+  if (m->err_host) cudaFreeHost(m->err_host);
+  if (m->own_stream && m->stream) cudaStreamDestroy(m->stream);
+  delete m;
+}
+
+bool is_device_pointer(const void* p) {
+  cudaPointerAttributes at{};
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+tvl_status launch(tvl_model* m, int token, int pos, int n_steps, int final_token) {
+  DecodeArgs a = m->args;
+  a.start_token = token;
+  a.start_pos = pos;
+  a.n_steps = n_steps;
+  a.final_token = final_token;
+  void* params[] = {&a};
+  TVL_CK(cudaLaunchCooperativeKernel((const void*)decode_kernel, dim3(a.G), dim3(kThreads), params,
+                                     (size_t)m->smem_bytes, m->stream));
+  return TVL_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, void* stream,
+                    tvl_model** out) {
+  if (out) *out = nullptr;
+  if (!out || !blob) {
+    set_error("tvl_load: null argument");
+    return TVL_E_INVAL;
+  }
+  if (!config_valid(cfg)) {
+    set_error("tvl_load: invalid configuration");
+    return TVL_E_INVAL;
+  }
+  const int d = cfg->dim, F = cfg->hidden_dim, H = cfg->n_heads, Hkv = cfg->n_kv_heads;
+  const int hd = d / H, kvd = Hkv * hd, V = cfg->vocab_size, S = cfg->max_seq, L = cfg->n_layers;
+  if (d % 32 != 0 || hd % 4 != 0 || hd > 256 || F % 4 != 0 || std::max(d, F) > 16384) {
+    set_error("tvl_load: the GPU path needs dim % 32 == 0, head_dim % 4 == 0 and <= 256, "
+              "hidden_dim % 4 == 0, max(dim, hidden_dim) <= 16384");
+    return TVL_E_UNSUPPORTED;
+  }
+  // §5.1 weight tying: explicit, or inferred from the blob size.
+  const size_t tied_bytes = (size_t)blob_layout(cfg, true).total;
+  const size_t untied_bytes = (size_t)blob_layout(cfg, false).total;
+  bool tied;
+  if (cfg->shared_classifier == 1) tied = true;
+  else if (cfg->shared_classifier == 0) tied = false;
+  else tied = blob_bytes < untied_bytes;
+  if (blob_bytes != (tied ? tied_bytes : untied_bytes)) {
+    set_error("tvl_load: blob_bytes " + std::to_string(blob_bytes) + " != expected " +
+              std::to_string(tied ? tied_bytes : untied_bytes));
+    return TVL_E_SIZE;
+  }
+  const BlobLayout bl = blob_layout(cfg, tied);
+  // the kernel streams [Wq|Wk|Wv] and [W1|W3] as single matrices
+  if (bl.wk != bl.wq + 4LL * d * d || bl.wv != bl.wk + 4LL * kvd * d ||
+      bl.w3 != bl.w1 + 4LL * F * d) {
+    set_error("tvl_load: layout has padding between fused matrices");
+    return TVL_E_UNSUPPORTED;
+  }
+
+  tvl_model* m = new (std::nothrow) tvl_model();
+  if (!m) return TVL_E_NOMEM;
+  m->cfg = *cfg;
+  m->tied = tied;
+  auto fail = [&](tvl_status s) {
+    destroy(m);
+    return s;
+  };
+  auto ck = [&](cudaError_t e, const char* what) -> tvl_status {
+    return e == cudaSuccess ? TVL_OK : cuda_fail(e, what);
+  };
+  tvl_status st;
+  if ((st = ck(cudaGetDevice(&m->device), "cudaGetDevice")) != TVL_OK) return fail(st);
+  int sms = 0, coop = 0, max_optin = 0;
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, m->device);
+  cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, m->device);
+  cudaDeviceGetAttribute(&max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, m->device);
+  if (!coop || sms <= 0) {
+    set_error("tvl_load: device lacks cooperative launch");
+    return fail(TVL_E_UNSUPPORTED);
+  }
+  const int G = sms;
+  const int nch_cap = nch_cap_for(S, H, G);
+  const SmemPlan sp = plan_smem(d, F, hd, H, nch_cap, max_optin);
+  if (sp.nst < 2) {
+    set_error("tvl_load: not enough shared memory for two weight stages");
+    return fail(TVL_E_UNSUPPORTED);
+  }
+  m->smem_bytes = sp.total;
+  if ((st = ck(cudaFuncSetAttribute((const void*)decode_kernel,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, sp.total),
+               "cudaFuncSetAttribute")) != TVL_OK)
+    return fail(st);
+  int per_sm = 0;
+  if ((st = ck(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, (const void*)decode_kernel,
+                                                              kThreads, sp.total),
+               "cudaOccupancyMaxActiveBlocksPerMultiprocessor")) != TVL_OK)
+    return fail(st);
+  if (per_sm < 1) {
+    set_error("tvl_load: decode kernel cannot be resident on an SM");
+    return fail(TVL_E_UNSUPPORTED);
+  }
+
+  // ---- arena: weights | rope | K cache | V cache | scratch -------------------------
+  const int att_stride = hd + 4;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = (size_t)a256((int64_t)(off + bytes));
+    return at;
+  };
+  const size_t o_w = take(blob_bytes);
+  const size_t o_rope = take((size_t)S * (hd / 2) * sizeof(float2));
+  const size_t kv_bytes = (size_t)std::max(L, 1) * S * kvd * 4;
+  const size_t o_kc = take(kv_bytes), o_vc = take(kv_bytes);
+  const size_t o_scr = off;
+  const size_t o_qkv = take(4ull * (d + 2 * kvd)), o_o = take(4ull * d), o_h13 = take(8ull * F);
+  const size_t o_f = take(4ull * d), o_lg = take(4ull * V);
+  const size_t o_att = take(4ull * H * nch_cap * att_stride);
+  const size_t o_cv = take(4ull * G), o_ci = take(4ull * G), o_tok = take(4ull * S);
+  const size_t o_ts = take(8ull * S), o_bar = take(8), o_err = take(4);
+  m->arena_bytes = off;
+  m->weight_bytes = blob_bytes;
+  if ((st = ck(cudaMalloc((void**)&m->arena, m->arena_bytes), "cudaMalloc(arena)")) != TVL_OK)
+    return fail(st);
+  if (stream) {
+    m->stream = (cudaStream_t)stream;
+  } else {
+    if ((st = ck(cudaStreamCreateWithFlags(&m->stream, cudaStreamNonBlocking),
+                 "cudaStreamCreate")) != TVL_OK)
+      return fail(st);
+    m->own_stream = true;
+  }
+  if ((st = ck(cudaHostAlloc((void**)&m->err_host, sizeof(int), cudaHostAllocMapped),
+               "cudaHostAlloc(err)")) != TVL_OK)
+    return fail(st);
+  *m->err_host = 0;
+  int* err_host_dev = nullptr;
+  if ((st = ck(cudaHostGetDevicePointer((void**)&err_host_dev, m->err_host, 0),
+               "cudaHostGetDevicePointer")) != TVL_OK)
+    return fail(st);
+
+  // ---- the single copy of the blob (pinned first, if it is not already) ------------
+  const bool dev_blob = is_device_pointer(blob);
+  bool registered = false;
+  if (!dev_blob) {
+    cudaPointerAttributes at{};
+    const bool pinned = cudaPointerGetAttributes(&at, blob) == cudaSuccess &&
+                        at.type == cudaMemoryTypeHost;
+    cudaGetLastError();
+    if (!pinned) {
+      int ro = 0;
+      cudaDeviceGetAttribute(&ro, cudaDevAttrHostRegisterReadOnlySupported, m->device);
+      unsigned flags = ro ? cudaHostRegisterReadOnly : cudaHostRegisterDefault;
+      registered = cudaHostRegister(const_cast<void*>(blob), blob_bytes, flags) == cudaSuccess;
+      if (!registered && ro)
+        registered =
+            cudaHostRegister(const_cast<void*>(blob), blob_bytes, cudaHostRegisterDefault) ==
+            cudaSuccess;
+      cudaGetLastError();  // an unpinnable blob is still copied, from pageable memory
+    }
+  }
+  st = ck(cudaMemcpyAsync(m->arena + o_w, blob, blob_bytes,
+                          dev_blob ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice, m->stream),
+          "cudaMemcpyAsync(blob)");
+  if (st == TVL_OK) st = ck(cudaStreamSynchronize(m->stream), "cudaStreamSynchronize(blob)");
+  if (registered) cudaHostUnregister(const_cast<void*>(blob));
+  if (st != TVL_OK) return fail(st);
+
+  // ---- RoPE table: pair i at position p turns by p * theta^(-2i/hd) ------------------
+  {
+    std::vector<float2> rope((size_t)S * (hd / 2));
+    for (int p = 0; p < S; ++p)
+      for (int i = 0; i < hd / 2; ++i) {
+        const double w = std::pow(cfg->rope_theta, -(2.0 * i) / (double)hd);
+        const double ang = (double)p * w;
+        rope[(size_t)p * (hd / 2) + i] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+      }
+    st = ck(cudaMemcpyAsync(m->arena + o_rope, rope.data(), rope.size() * sizeof(float2),
+                            cudaMemcpyHostToDevice, m->stream),
+            "cudaMemcpyAsync(rope)");
+    if (st == TVL_OK)
+      st = ck(cudaMemsetAsync(m->arena + o_kc, 0, m->arena_bytes - o_kc, m->stream),
+              "cudaMemsetAsync(state)");
+    if (st == TVL_OK) st = ck(cudaStreamSynchronize(m->stream), "cudaStreamSynchronize(rope)");
+    if (st != TVL_OK) return fail(st);
+  }
+  (void)o_scr;
+
+  // ---- kernel arguments that do not change between launches --------------------------
+  DecodeArgs& a = m->args;
+  unsigned char* W = m->arena + o_w;
+  a.E = reinterpret_cast<const float*>(W + bl.E);
+  a.g_final = reinterpret_cast<const float*>(W + bl.g_final);
+  a.Wcls = reinterpret_cast<const float*>(W + (tied ? bl.E : bl.Wcls));
+  a.layer0 = W + bl.l0;
+  a.layer_stride = bl.stride;
+  a.o_gatt = bl.g_att;
+  a.o_wqkv = bl.wq;
+  a.o_wo = bl.wo;
+  a.o_gffn = bl.g_ffn;
+  a.o_w13 = bl.w1;
+  a.o_w2 = bl.w2;
+  a.rope = reinterpret_cast<const float2*>(m->arena + o_rope);
+  a.kc = reinterpret_cast<float*>(m->arena + o_kc);
+  a.vc = reinterpret_cast<float*>(m->arena + o_vc);
+  a.qkv = reinterpret_cast<float*>(m->arena + o_qkv);
+  a.o_out = reinterpret_cast<float*>(m->arena + o_o);
+  a.h13 = reinterpret_cast<float*>(m->arena + o_h13);
+  a.f_out = reinterpret_cast<float*>(m->arena + o_f);
+  a.logits = reinterpret_cast<float*>(m->arena + o_lg);
+  a.att = reinterpret_cast<float*>(m->arena + o_att);
+  a.cand_val = reinterpret_cast<float*>(m->arena + o_cv);
+  a.cand_idx = reinterpret_cast<int*>(m->arena + o_ci);
+  a.tokens = reinterpret_cast<int*>(m->arena + o_tok);
+  a.ts = reinterpret_cast<unsigned long long*>(m->arena + o_ts);
+  a.bar = reinterpret_cast<unsigned long long*>(m->arena + o_bar);
+  a.err = reinterpret_cast<int*>(m->arena + o_err);
+  a.err_host = err_host_dev;
+  a.d = d; a.F = F; a.V = V; a.L = L; a.H = H; a.Hkv = Hkv; a.hd = hd; a.kvd = kvd; a.S = S;
+  a.G = G;
+  a.att_stride = att_stride;
+  a.nch_cap = nch_cap;
+  a.eps = (float)cfg->norm_eps;
+  a.att_scale = (float)(1.0 / std::sqrt((double)hd));
+  a.nst = sp.nst;
+  a.sm_ring = sp.ring; a.sm_bars = sp.bars; a.sm_xs = sp.xs; a.sm_vec = sp.vec;
+  a.sm_pdot = sp.pdot; a.sm_att = sp.att; a.sm_misc = sp.misc;
+  a.barrier_limit_ns = kWaitLimitNs;
+  m->streamed_bytes =
+      4LL * ((int64_t)L * ((int64_t)(d + 2 * kvd) * d + (int64_t)d * d + 3LL * F * d + 2LL * d) +
+             (int64_t)V * d + 2LL * d);
+  *out = m;
+  return TVL_OK;
+}
+
+tvl_status tvl_load_file(const tvl_config* cfg, const char* path, void* stream, tvl_model** out) {
+  if (out) *out = nullptr;
+  if (!path || !out) {
+    set_error("tvl_load_file: null argument");
+    return TVL_E_INVAL;
+  }
+  const int fd = open(path, O_RDONLY);
+  if (fd < 0) {
+    set_error(std::string("tvl_load_file: cannot open ") + path);
+    return TVL_E_INVAL;
+  }
+  struct stat sb;
+  if (fstat(fd, &sb) != 0 || sb.st_size <= 0) {
+    close(fd);
+    set_error("tvl_load_file: cannot stat file");
+    return TVL_E_INVAL;
+  }
+  int flags = MAP_PRIVATE;
+#ifdef MAP_POPULATE
+  flags |= MAP_POPULATE;  // pre-fault the pages (the paper's Linux hint)
+#endif
+  void* p = mmap(nullptr, (size_t)sb.st_size, PROT_READ, flags, fd, 0);
+  close(fd);
+  if (p == MAP_FAILED) {
+    set_error("tvl_load_file: mmap failed");
+    return TVL_E_NOMEM;
+  }
+  const tvl_status st = tvl_load(cfg, p, (size_t)sb.st_size, stream, out);
+  munmap(p, (size_t)sb.st_size);
+  return st;
+}
+
+tvl_status tvl_forward(tvl_model* m, int32_t token, int32_t pos, float* logits_out) {
+  if (!m) {
+    set_error("tvl_forward: null model");
+    return TVL_E_INVAL;
+  }
+  if (m->sticky != TVL_OK) return m->sticky;
+  if (token < 0 || token >= m->cfg.vocab_size || pos < 0 || pos >= m->cfg.max_seq) {
+    set_error("tvl_forward: token or position out of range");
+    return TVL_E_RANGE;
+  }
+  tvl_status st = launch(m, token, pos, 1, 0);
+  if (st != TVL_OK) return st;
+  if (!logits_out) return TVL_OK;
+  const size_t bytes = (size_t)m->cfg.vocab_size * 4;
+  if (is_device_pointer(logits_out)) {
+    TVL_CK(cudaMemcpyAsync(logits_out, m->args.logits, bytes, cudaMemcpyDeviceToDevice,
+                           m->stream));
+    return TVL_OK;
+  }
+  TVL_CK(cudaMemcpyAsync(logits_out, m->args.logits, bytes, cudaMemcpyDeviceToHost, m->stream));
+  TVL_CK(cudaStreamSynchronize(m->stream));
+  return check_device_error(m);
+}
+
+tvl_status tvl_decode_greedy(tvl_model* m, int32_t start_token, int32_t start_pos,
+                             int32_t n_steps, int32_t* tokens_out) {
+  if (!m) {
+    set_error("tvl_decode_greedy: null model");
+    return TVL_E_INVAL;
+  }
+  if (m->sticky != TVL_OK) return m->sticky;
+  if (start_token < 0 || start_token >= m->cfg.vocab_size || start_pos < 0 || n_steps < 1 ||
+      (int64_t)start_pos + n_steps > m->cfg.max_seq) {
+    set_error("tvl_decode_greedy: token, position or step count out of range");
+    return TVL_E_RANGE;
+  }
+  tvl_status st = launch(m, start_token, start_pos, n_steps, 1);
+  if (st != TVL_OK) return st;
+  if (!tokens_out) return TVL_OK;
+  TVL_CK(cudaMemcpyAsync(tokens_out, m->args.tokens, 4ull * n_steps, cudaMemcpyDeviceToHost,
+                         m->stream));
+  TVL_CK(cudaStreamSynchronize(m->stream));
+  return check_device_error(m);
+}
+
+tvl_status tvl_sync(tvl_model* m) {
+  if (!m) {
+    set_error("tvl_sync: null model");
+    return TVL_E_INVAL;
+  }
+  TVL_CK(cudaStreamSynchronize(m->stream));
+  if (m->sticky != TVL_OK) return m->sticky;
+  return check_device_error(m);
+}
+
+void tvl_free(tvl_model* m) {
+  if (!m) return;
+  if (m->stream) cudaStreamSynchronize(m->stream);
+  destroy(m);
+}
+
+tvl_status tvl_get_info(const tvl_model* m, tvl_model_info* out) {
+  if (!m || !out) {
+    set_error("tvl_get_info: null argument");
+    return TVL_E_INVAL;
+  }
+  out->arena_bytes = (int64_t)m->arena_bytes;
+  out->weight_bytes = (int64_t)m->weight_bytes;
+  out->streamed_bytes = m->streamed_bytes;
+  out->grid = m->args.G;
+  out->threads = kThreads;
+  out->smem_bytes = m->smem_bytes;
+  out->ring_stages = m->args.nst;
+  out->stage_bytes = kStageBytes;
+  out->tied = m->tied ? 1 : 0;
+  out->barriers_per_step = 5 * m->cfg.n_layers + 1;
+  return TVL_OK;
+}
+
+tvl_status tvl_step_times(tvl_model* m, uint64_t* ns_out, int32_t n) {
+  if (!m || !ns_out || n < 1 || n > m->cfg.max_seq) {
+    set_error("tvl_step_times: bad argument");
+    return TVL_E_INVAL;
+  }
+  TVL_CK(cudaMemcpyAsync(ns_out, m->args.ts, 8ull * n, cudaMemcpyDeviceToHost, m->stream));
+  TVL_CK(cudaStreamSynchronize(m->stream));
+  return TVL_OK;
+}
+
+tvl_status tvl_selftest_barrier_timeout(int32_t limit_ms) {
+  if (limit_ms < 1 || limit_ms > 10000) {
+    set_error("tvl_selftest_barrier_timeout: limit_ms out of [1, 10000]");
+    return TVL_E_INVAL;
+  }
+  unsigned char* buf = nullptr;
+  TVL_CK(cudaMalloc((void**)&buf, 256));
+  tvl_status st = TVL_OK;
+  cudaError_t e = cudaMemset(buf, 0, 256);
+  DecodeArgs a{};
+  a.bar = reinterpret_cast<unsigned long long*>(buf);
+  a.err = reinterpret_cast<int*>(buf + 64);
+  a.err_host = nullptr;
+  a.G = 1;
+  a.barrier_limit_ns = (unsigned long long)limit_ms * 1000000ull;
+  if (e == cudaSuccess) {
+    barrier_selftest_kernel<<<1, kThreads>>>(a);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  int code = 0;
+  if (e == cudaSuccess) e = cudaMemcpy(&code, buf + 64, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) st = cuda_fail(e, "barrier self-test");
+  cudaFree(buf);
+  if (st != TVL_OK) return st;
+  if (code == 0) {
+    set_error("barrier self-test: the wait did not report a timeout");
+    return TVL_E_CUDA;
+  }
+  set_error("barrier self-test: the bounded wait expired as intended");
+  return (tvl_status)code;
+}
+
+}  // extern "C"

@@ -1,0 +1,222 @@
+// gemv.cu — standalone y = W x (paper §6.1) on the weight-streaming engine.
+//
+// One CTA per SM streams its contiguous share of W through the shared-memory
+// stage ring. Matrices with few rows are split along K into S chunks so that
+// every SM gets work: virtual row v = (row v / S, chunk v % S); each virtual
+// row's partial lands in a scratch buffer, and each row is summed over its
+// S chunks in chunk order — by the CTA that owns the whole row, or for a row
+// shared by two CTAs, by whichever of them finishes last (a per-row arrival
+// counter). The result does not depend on timing. Every wait in the kernel is
+// bounded (one second); a CTA whose stage never lands leaves early, which
+// only a broken device can cause.
+#include <map>
+#include <mutex>
+#include <utility>
+
+#include "host_common.h"
+#include "stream_gemv.cuh"
+
+using namespace tvl;
+
+namespace tvl {
+
+struct GemvArgs {
+  const float* W;
+  const float* x;
+  float* y;
+  int M, K, S, Kc;
+  long long nv;  // virtual rows = M * S
+  float* part;   // [M * S] when S > 1
+  int* cnt;      // [M], zero between calls
+  int nst;
+  int sm_ring, sm_bars, sm_x, sm_pdot, sm_misc;
+};
+
+struct EpiPart {
+  float* part;
+  __device__ __forceinline__ void store(int v, float val) { part[v] = val; }
+};
+
+__global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const GemvArgs a) {
+  extern __shared__ __align__(128) unsigned char smem[];
+  Ring r;
+  r.buf = smem + a.sm_ring;
+  r.full = reinterpret_cast<uint64_t*>(smem + a.sm_bars);
+  r.empty = r.full + a.nst;
+  r.nst = a.nst;
+  volatile int* s_abort = reinterpret_cast<volatile int*>(smem + a.sm_misc);
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < a.nst; ++i) {
+      mbar_init(&r.full[i], 1);
+      mbar_init(&r.empty[i], 1);
+    }
+    *s_abort = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  const StagePlan p = plan_stages(a.nv, a.Kc, gridDim.x, blockIdx.x);
+  uint32_t g = 0;
+  if (threadIdx.x >= kConsumerThreads) {
+    if (threadIdx.x == kConsumerThreads) {
+      produce_phase(r, g, a.W, p, l2_evict_first(), nullptr, nullptr, s_abort);
+      drain_ring(r, g);
+    }
+    return;
+  }
+  float* xs = reinterpret_cast<float*>(smem + a.sm_x);
+  float* pdot = reinterpret_cast<float*>(smem + a.sm_pdot);
+  const float4* x4 = reinterpret_cast<const float4*>(a.x);
+  for (int j = threadIdx.x; j < (a.K >> 2); j += kConsumerThreads)
+    reinterpret_cast<float4*>(xs)[j] = __ldg(x4 + j);
+  named_bar_sync(kBarConsumers, kConsumerThreads);
+  if (a.S == 1) {
+    EpiStore e{a.y};
+    consume_phase(r, g, p, xs, 1, a.Kc, pdot, e, nullptr, nullptr, s_abort);
+    return;
+  }
+  EpiPart e{a.part};
+  if (!consume_phase(r, g, p, xs, a.S, a.Kc, pdot, e, nullptr, nullptr, s_abort)) return;
+  if (p.r1 <= p.r0) return;
+  named_bar_sync(kBarConsumers, kConsumerThreads);
+  const int S = a.S;
+  const int ra = p.r0 / S, rb = (p.r1 - 1) / S;
+  for (int row = ra + threadIdx.x; row <= rb; row += kConsumerThreads) {
+    const int lo = max(p.r0, row * S), hi = min(p.r1, (row + 1) * S);
+    const int mine = hi - lo;
+    bool last = (mine == S);
+    if (!last) {
+      __threadfence();
+      const int before = atomicAdd(a.cnt + row, mine);
+      last = (before + mine == S);
+      if (last) __threadfence();
+    }
+    if (last) {
+      float v = 0.f;
+      for (int s = 0; s < S; ++s) v += __ldcg(a.part + (size_t)row * S + s);
+      a.y[row] = v;
+      if (mine != S) a.cnt[row] = 0;
+    }
+  }
+}
+
+// Any shape or alignment: one warp per row, scalar loads.
+__global__ void gemv_rowwise_kernel(const float* __restrict__ W, const float* __restrict__ x,
+                                    float* __restrict__ y, int M, int K) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (warp >= M) return;
+  const float* w = W + (size_t)warp * K;
+  float acc = 0.f;
+  for (int j = lane; j < K; j += 32) acc = fmaf(__ldg(w + j), __ldg(x + j), acc);
+  acc = warp_sum(acc);
+  if (lane == 0) y[warp] = acc;
+}
+
+}  // namespace tvl
+
+namespace {
+
+struct Workspace {
+  float* part = nullptr;
+  int* cnt = nullptr;
+  long long part_cap = 0;
+  int cnt_cap = 0;
+};
+
+std::mutex g_ws_mu;
+std::map<std::pair<int, cudaStream_t>, Workspace> g_ws;
+
+struct DevInfo {
+  int sms = 0, max_optin = 0;
+  bool attr_set = false;
+};
+std::map<int, DevInfo> g_dev;
+
+int split_for(int M, int K, int G) {
+  int S = 1;
+  while ((long long)M * S < 16LL * G && K % (8 * S) == 0 && K / (2 * S) >= 128) S *= 2;
+  return S;
+}
+
+}  // namespace
+
+extern "C" tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t d_out,
+                               int32_t d_in, void* stream) {
+  if (!W || !x || !y || d_out < 1 || d_in < 1) {
+    set_error("tvl_gemv: null pointer or non-positive size");
+    return TVL_E_INVAL;
+  }
+  cudaStream_t s = (cudaStream_t)stream;
+  int dev = 0;
+  TVL_CK(cudaGetDevice(&dev));
+  DevInfo info;
+  {
+    std::lock_guard<std::mutex> lk(g_ws_mu);
+    DevInfo& di = g_dev[dev];
+    if (di.sms == 0) {
+      cudaDeviceGetAttribute(&di.sms, cudaDevAttrMultiProcessorCount, dev);
+      cudaDeviceGetAttribute(&di.max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    }
+    info = di;
+  }
+  const bool aligned = ((uintptr_t)W % 16 == 0) && ((uintptr_t)x % 16 == 0) && d_in % 4 == 0;
+  if (!aligned || d_in > 16384) {
+    const int threads = 256, rows_per_block = threads / 32;
+    gemv_rowwise_kernel<<<(d_out + rows_per_block - 1) / rows_per_block, threads, 0, s>>>(
+        W, x, y, d_out, d_in);
+    TVL_CK(cudaGetLastError());
+    return TVL_OK;
+  }
+  GemvArgs a{};
+  a.W = W;
+  a.x = x;
+  a.y = y;
+  a.M = d_out;
+  a.K = d_in;
+  a.S = split_for(d_out, d_in, info.sms);
+  a.Kc = d_in / a.S;
+  a.nv = (long long)d_out * a.S;
+  const int G = (int)(a.nv < info.sms ? a.nv : info.sms);
+  // shared memory: ring | barriers | x | piece sums | misc
+  const int xbytes = (int)a128(4LL * d_in), pdot = 2 * kMaxPieces * 4, bars = 128, misc = 128;
+  int nst = (info.max_optin - xbytes - pdot - bars - misc) / kStageBytes;
+  if (nst > 6) nst = 6;
+  if (nst < 2) {
+    set_error("tvl_gemv: not enough shared memory");
+    return TVL_E_UNSUPPORTED;
+  }
+  a.nst = nst;
+  a.sm_ring = 0;
+  a.sm_bars = nst * kStageBytes;
+  a.sm_x = a.sm_bars + bars;
+  a.sm_pdot = a.sm_x + xbytes;
+  a.sm_misc = a.sm_pdot + pdot;
+  const int smem = a.sm_misc + misc;
+  {
+    std::lock_guard<std::mutex> lk(g_ws_mu);
+    Workspace& ws = g_ws[{dev, s}];
+    const long long need_part = a.S > 1 ? a.nv : 1;
+    const int need_cnt = a.S > 1 ? d_out : 1;
+    if (ws.part_cap < need_part || ws.cnt_cap < need_cnt || !ws.part) {
+      if (ws.part) {  // earlier kernels on this stream may still use the old buffers
+        TVL_CK(cudaStreamSynchronize(s));
+        cudaFree(ws.part);
+        cudaFree(ws.cnt);
+        ws = Workspace{};
+      }
+      const long long pc = need_part > 4096 ? need_part : 4096;
+      const int cc = need_cnt > 4096 ? need_cnt : 4096;
+      TVL_CK(cudaMalloc((void**)&ws.part, 4 * pc + 256));
+      TVL_CK(cudaMalloc((void**)&ws.cnt, 4LL * cc + 256));
+      TVL_CK(cudaMemsetAsync(ws.cnt, 0, 4LL * cc + 256, s));
+      ws.part_cap = pc;
+      ws.cnt_cap = cc;
+    }
+    a.part = ws.part;
+    a.cnt = ws.cnt;
+  }
+  TVL_CK(cudaFuncSetAttribute((const void*)gemv_stream_kernel,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+  gemv_stream_kernel<<<G, kThreads, smem, s>>>(a);
+  TVL_CK(cudaGetLastError());
+  return TVL_OK;
+}

@@ -1,0 +1,178 @@
+"""Decode step on the GPU (persistent kernel through the C ABI) vs the CPU oracle.
+
+Teacher forcing: both sides are fed the oracle's greedy tokens and every
+step's logits are compared (max |d| <= 2e-3 * max |logit|). The device-side
+greedy loop (tvl_decode_greedy, the launch the benchmark times) must produce
+the oracle's tokens wherever the oracle's top-2 margin exceeds 1e-2.
+"""
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from helpers import (assert_logits_close, compare_greedy, lockstep_greedy, small_config,
+                     teacher_forced)
+from paper_2601_03324_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def tvl():
+    from paper_2601_03324_gb300 import tvl as t
+    return t
+
+
+def check_model(tvl, cfg, blob, n_steps, start=1, greedy=True, check_every=1, label=""):
+    ref = oracle.Model(cfg, blob, 64)
+    with tvl.Model(cfg, blob) as m:
+        toks, ref_logits, worst = lockstep_greedy(m, ref, start, n_steps,
+                                                  check_every=check_every, label=label)
+        if greedy:
+            gen = m.decode_greedy(start, 0, n_steps)
+            compare_greedy(gen, toks[1:] + [int(np.argmax(ref_logits[-1]))], ref_logits)
+    return worst
+
+
+def test_tiny_model_64_steps(tvl):
+    cfg = synth.model_config("tiny")
+    blob = synth.make_blob(cfg)
+    check_model(tvl, cfg, blob, cfg["steps"], label="tiny")
+
+
+@pytest.mark.parametrize("kw", [
+    dict(),                                    # several layers, multi-chunk attention
+    dict(n_kv_heads=2),                        # grouped query heads (2 query heads per kv head)
+    dict(n_kv_heads=1, n_heads=8),             # one kv head, head_dim 8
+    dict(n_layers=0),                          # embedding -> final norm -> classifier
+    dict(n_layers=1, hidden_dim=36, dim=32, n_heads=1, vocab_size=7),  # tiny vocab, one head
+    dict(dim=96, n_heads=2, hidden_dim=8200, vocab_size=333),          # W2 rows span two stages
+    dict(dim=128, n_heads=1, hidden_dim=256),  # head_dim 128
+], ids=["base", "gqa2", "mqa", "L0", "v7", "wide_ffn", "hd128"])
+def test_small_shapes_match_oracle(tvl, kw):
+    cfg = small_config(**kw)
+    blob = synth.make_blob(cfg, seed=21)
+    check_model(tvl, cfg, blob, cfg["max_seq"], label=str(kw))
+
+
+def test_tied_classifier_inferred_from_blob_size(tvl):
+    cfg = small_config(shared_classifier=-1)
+    blob = synth.make_blob(cfg, seed=5, tied=True)
+    with tvl.Model(cfg, blob) as m:
+        assert m.info().tied == 1
+    check_model(tvl, cfg, blob, 16, greedy=False)
+
+
+def test_positions_beyond_one_attention_chunk_limit(tvl):
+    # 128 heads leave one attention item per head until position 1023 (chunks
+    # of up to 1024 positions); later positions need two chunks per head.
+    cfg = small_config(n_layers=1, dim=512, n_heads=128, n_kv_heads=64, vocab_size=300,
+                       max_seq=1100, hidden_dim=64)
+    blob = synth.make_blob(cfg, seed=8)
+    toks = synth.uniform_ints(1100, 8, 1, 0, 299)
+    ref = oracle.Model(cfg, blob, 64)
+    with tvl.Model(cfg, blob) as m:
+        teacher_forced(m, ref, toks, check_every=37, label="long")
+
+
+def test_device_logits_pointer_and_repeat_are_bitwise_stable(tvl):
+    cfg = small_config()
+    blob = synth.make_blob(cfg, seed=2)
+    with tvl.Model(cfg, blob) as m:
+        dl = torch.empty(cfg["vocab_size"], device="cuda")
+        h1 = np.empty(cfg["vocab_size"], np.float32)
+        m.forward(3, 0, h1)
+        m.forward(3, 0, dl.data_ptr())
+        m.sync()
+        assert np.array_equal(dl.cpu().numpy(), h1)
+
+
+def test_out_of_range_arguments(tvl):
+    cfg = small_config(max_seq=8)
+    blob = synth.make_blob(cfg, seed=2)
+    with tvl.Model(cfg, blob) as m:
+        for tok, pos in ((cfg["vocab_size"], 0), (-1, 0), (0, 8), (0, -1)):
+            with pytest.raises(tvl.TvlError) as e:
+                m.forward(tok, pos)
+            assert e.value.status == tvl.E_RANGE
+        with pytest.raises(tvl.TvlError) as e:
+            m.decode_greedy(1, 4, 5)
+        assert e.value.status == tvl.E_RANGE
+        m.decode_greedy(1, 4, 4)  # the boundary case fits
+
+
+def test_load_file_equals_load(tvl, tmp_path):
+    cfg = small_config()
+    blob = synth.make_blob(cfg, seed=4)
+    path = os.path.join(tmp_path, "model.tvl")
+    blob.tofile(path)
+    a = np.empty(cfg["vocab_size"], np.float32)
+    b = np.empty_like(a)
+    with tvl.Model(cfg, blob) as m:
+        m.forward(7, 0, a)
+    with tvl.Model(cfg, path=path) as m:
+        m.forward(7, 0, b)
+    assert np.array_equal(a, b)
+    with pytest.raises(tvl.TvlError) as e:
+        tvl.Model(cfg, blob[:-32])
+    assert e.value.status == tvl.E_SIZE
+
+
+def test_barrier_timeout_is_reported_and_context_survives(tvl):
+    assert tvl.tvl_selftest_barrier_timeout(50) == tvl.E_TIMEOUT
+    cfg = small_config(n_layers=1)
+    blob = synth.make_blob(cfg, seed=1)
+    ref = oracle.Model(cfg, blob, 64)
+    out = np.empty(cfg["vocab_size"], np.float32)
+    with tvl.Model(cfg, blob) as m:
+        m.forward(1, 0, out)
+    assert_logits_close(out, ref.forward(1, 0), "after timeout test")
+
+
+def test_110m_model_256_greedy_steps(tvl):
+    """The benchmark's workload: the 110M shape, 256 steps from token 1."""
+    cfg = synth.model_config("110m")
+    blob = synth.make_blob(cfg)
+    worst = check_model(tvl, cfg, blob, cfg["steps"], check_every=1, label="110m")
+    assert worst <= 2e-3
+
+
+def test_110m_long_context_fill_then_greedy(tvl):
+    """896 random prompt tokens fed one step at a time, then 128 greedy steps."""
+    cfg = synth.model_config("110m")
+    blob = synth.make_blob(cfg)
+    prompt = synth.long_context_tokens(896)
+    ref = oracle.Model(cfg, blob, 64)
+    with tvl.Model(cfg, blob) as m:
+        teacher_forced(m, ref, prompt, check_every=64, label="110m fill")
+        # continue greedily on both sides from the last prompt logits
+        lg = ref.forward(int(prompt[-1]), 895)  # recompute position 895 (same cache contents)
+        start = int(np.argmax(lg))
+        toks, ref_logits = ref.greedy(start, 128, start_pos=896)
+        gen = m.decode_greedy(start, 896, 128)
+        agreed = compare_greedy(gen, toks[1:] + [int(np.argmax(ref_logits[-1]))], ref_logits)
+        if agreed == 128:  # same tokens in the cache on both sides
+            out = np.empty(cfg["vocab_size"], np.float32)
+            m.forward(toks[-1], 1023, out)  # last position, full 1024-entry cache
+            assert_logits_close(out, ref_logits[-1], "110m pos 1023")
+
+
+def test_7b_shape_teacher_forced_and_greedy(tvl):
+    """7B shape (~27 GB of weights): a few teacher-forced steps checked against
+    the oracle, then the 16-step device greedy run checked where it can be."""
+    cfg = synth.model_config("7b")
+    free, total = torch.cuda.mem_get_info()
+    if free < 32e9:
+        pytest.skip("needs ~32 GB of free device memory")
+    blob = synth.make_blob(cfg)
+    ref = oracle.Model(cfg, blob, 64)
+    n_ref = 3
+    with tvl.Model(cfg, blob) as m:
+        toks, ref_logits, _ = lockstep_greedy(m, ref, 1, n_ref, label="7b")
+        gen = m.decode_greedy(1, 0, cfg["steps"])
+        nxt = int(np.argmax(ref_logits[-1]))
+        compare_greedy(gen[:n_ref], toks[1:] + [nxt], ref_logits)
+        assert gen.min() >= 0 and gen.max() < cfg["vocab_size"]
