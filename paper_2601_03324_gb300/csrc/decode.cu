@@ -29,6 +29,7 @@ struct tvl_model {
   DecodeArgs args{};
   int smem_bytes = 0;
   int* err_host = nullptr;  // pinned, mapped: the kernel writes its error code here too
+  unsigned epoch = 1;       // tag of the next launch's first exchange (0 = never written)
   tvl_status sticky = TVL_OK;
 };
 
@@ -44,8 +45,8 @@ SmemPlan plan_smem(int d, int F, int hd, int H, int nch_cap, int max_bytes) {
       std::max(3 * hd + kAttMaxChunk + 4 * kConsumerThreads, 2 * H * nch_cap) + 16;
   const int xs = (int)a128(4LL * d), vec = (int)a128(4LL * std::max(d, F));
   const int pdot = 2 * kMaxPieces * 4, att = (int)a128(4LL * att_floats), misc = 256;
-  const int bars = 2 * 8 * 8;
-  const int other = bars + xs + vec + pdot + att + misc;
+  const int bars = 8 * 8;
+  const int other = bars + xs + vec + pdot + att + misc + 1024;  // + static shared memory
   int nst = (max_bytes - other) / kStageBytes;
   if (nst > 8) nst = 8;
   p.nst = nst;
@@ -82,7 +83,7 @@ tvl_status check_device_error(tvl_model* m) {
   const int code = *reinterpret_cast<volatile int*>(m->err_host);
   if (code != 0) {
     m->sticky = (tvl_status)code;
-    set_error("a bounded device-side wait expired (grid barrier or stage copy); "
+    set_error("a bounded device-side wait expired (exchange poll or stage copy); "
               "the model's device state is no longer consistent");
     return m->sticky;
   }
@@ -112,9 +113,12 @@ tvl_status launch(tvl_model* m, int token, int pos, int n_steps, int final_token
   a.start_pos = pos;
   a.n_steps = n_steps;
   a.final_token = final_token;
+  a.epoch0 = m->epoch;
   void* params[] = {&a};
   TVL_CK(cudaLaunchCooperativeKernel((const void*)decode_kernel, dim3(a.G), dim3(kThreads), params,
                                      (size_t)m->smem_bytes, m->stream));
+  // tags wrap modulo 2^32; a stale word is never within one launch of a live tag
+  m->epoch += (unsigned)n_steps * (unsigned)(kPhasesPerLayer * m->cfg.n_layers + 1);
   return TVL_OK;
 }
 
@@ -216,11 +220,11 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   const size_t kv_bytes = (size_t)std::max(L, 1) * S * kvd * 4;
   const size_t o_kc = take(kv_bytes), o_vc = take(kv_bytes);
   const size_t o_scr = off;
-  const size_t o_qkv = take(4ull * (d + 2 * kvd)), o_o = take(4ull * d), o_h13 = take(8ull * F);
-  const size_t o_f = take(4ull * d), o_lg = take(4ull * V);
-  const size_t o_att = take(4ull * H * nch_cap * att_stride);
-  const size_t o_cv = take(4ull * G), o_ci = take(4ull * G), o_tok = take(4ull * S);
-  const size_t o_ts = take(8ull * S), o_bar = take(8), o_err = take(4);
+  const size_t o_qkv = take(8ull * (d + 2 * kvd)), o_o = take(8ull * d), o_h13 = take(16ull * F);
+  const size_t o_f = take(8ull * d), o_lg = take(4ull * V);
+  const size_t o_att = take(8ull * H * nch_cap * att_stride);
+  const size_t o_cand = take(8ull * 2 * G * 2), o_tok = take(4ull * S);
+  const size_t o_ts = take(8ull * S), o_err = take(4);
   m->arena_bytes = off;
   m->weight_bytes = blob_bytes;
   if ((st = ck(cudaMalloc((void**)&m->arena, m->arena_bytes), "cudaMalloc(arena)")) != TVL_OK)
@@ -306,17 +310,15 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   a.rope = reinterpret_cast<const float2*>(m->arena + o_rope);
   a.kc = reinterpret_cast<float*>(m->arena + o_kc);
   a.vc = reinterpret_cast<float*>(m->arena + o_vc);
-  a.qkv = reinterpret_cast<float*>(m->arena + o_qkv);
-  a.o_out = reinterpret_cast<float*>(m->arena + o_o);
-  a.h13 = reinterpret_cast<float*>(m->arena + o_h13);
-  a.f_out = reinterpret_cast<float*>(m->arena + o_f);
+  a.x_qkv = reinterpret_cast<unsigned long long*>(m->arena + o_qkv);
+  a.x_o = reinterpret_cast<unsigned long long*>(m->arena + o_o);
+  a.x_h13 = reinterpret_cast<unsigned long long*>(m->arena + o_h13);
+  a.x_f = reinterpret_cast<unsigned long long*>(m->arena + o_f);
   a.logits = reinterpret_cast<float*>(m->arena + o_lg);
-  a.att = reinterpret_cast<float*>(m->arena + o_att);
-  a.cand_val = reinterpret_cast<float*>(m->arena + o_cv);
-  a.cand_idx = reinterpret_cast<int*>(m->arena + o_ci);
+  a.x_att = reinterpret_cast<unsigned long long*>(m->arena + o_att);
+  a.x_cand = reinterpret_cast<unsigned long long*>(m->arena + o_cand);
   a.tokens = reinterpret_cast<int*>(m->arena + o_tok);
   a.ts = reinterpret_cast<unsigned long long*>(m->arena + o_ts);
-  a.bar = reinterpret_cast<unsigned long long*>(m->arena + o_bar);
   a.err = reinterpret_cast<int*>(m->arena + o_err);
   a.err_host = err_host_dev;
   a.d = d; a.F = F; a.V = V; a.L = L; a.H = H; a.Hkv = Hkv; a.hd = hd; a.kvd = kvd; a.S = S;
@@ -328,7 +330,7 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   a.nst = sp.nst;
   a.sm_ring = sp.ring; a.sm_bars = sp.bars; a.sm_xs = sp.xs; a.sm_vec = sp.vec;
   a.sm_pdot = sp.pdot; a.sm_att = sp.att; a.sm_misc = sp.misc;
-  a.barrier_limit_ns = kWaitLimitNs;
+  a.wait_limit_ns = kWaitLimitNs;
   m->streamed_bytes =
       4LL * ((int64_t)L * ((int64_t)(d + 2 * kvd) * d + (int64_t)d * d + 3LL * F * d + 2LL * d) +
              (int64_t)V * d + 2LL * d);
@@ -443,7 +445,7 @@ tvl_status tvl_get_info(const tvl_model* m, tvl_model_info* out) {
   out->ring_stages = m->args.nst;
   out->stage_bytes = kStageBytes;
   out->tied = m->tied ? 1 : 0;
-  out->barriers_per_step = 5 * m->cfg.n_layers + 1;
+  out->barriers_per_step = kPhasesPerLayer * m->cfg.n_layers + 1;
   return TVL_OK;
 }
 
@@ -465,28 +467,24 @@ tvl_status tvl_selftest_barrier_timeout(int32_t limit_ms) {
   unsigned char* buf = nullptr;
   TVL_CK(cudaMalloc((void**)&buf, 256));
   tvl_status st = TVL_OK;
-  cudaError_t e = cudaMemset(buf, 0, 256);
-  DecodeArgs a{};
-  a.bar = reinterpret_cast<unsigned long long*>(buf);
-  a.err = reinterpret_cast<int*>(buf + 64);
-  a.err_host = nullptr;
-  a.G = 1;
-  a.barrier_limit_ns = (unsigned long long)limit_ms * 1000000ull;
+  cudaError_t e = cudaMemset(buf, 0, 256);  // tag 0: never the awaited tag 1
   if (e == cudaSuccess) {
-    barrier_selftest_kernel<<<1, kThreads>>>(a);
+    wait_selftest_kernel<<<1, kThreads>>>(reinterpret_cast<unsigned long long*>(buf),
+                                          reinterpret_cast<int*>(buf + 64),
+                                          (unsigned long long)limit_ms * 1000000ull);
     e = cudaGetLastError();
   }
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
   int code = 0;
   if (e == cudaSuccess) e = cudaMemcpy(&code, buf + 64, sizeof(int), cudaMemcpyDeviceToHost);
-  if (e != cudaSuccess) st = cuda_fail(e, "barrier self-test");
+  if (e != cudaSuccess) st = cuda_fail(e, "wait self-test");
   cudaFree(buf);
   if (st != TVL_OK) return st;
   if (code == 0) {
-    set_error("barrier self-test: the wait did not report a timeout");
+    set_error("wait self-test: the wait did not report a timeout");
     return TVL_E_CUDA;
   }
-  set_error("barrier self-test: the bounded wait expired as intended");
+  set_error("wait self-test: the bounded wait expired as intended");
   return (tvl_status)code;
 }
 

@@ -1,9 +1,8 @@
 // decode_kernel.cuh — one persistent kernel runs whole decode steps of a
 // Llama-2-architecture decoder (paper §2.1, §7.1), one CTA per SM.
 //
-// Per step and layer the consumer warps of every CTA run five phases, each
-// ended by a grid-wide barrier (every phase needs all outputs of the one
-// before):
+// Per step and layer the consumer warps of every CTA run five phases; each
+// needs all outputs of the phase before:
 //   1. x_b = RMSNorm(x, g_att); [q|k|v] = Wqkv x_b         (rows split over CTAs)
 //   2. RoPE on q, k; k, v into the cache; attention partials per
 //      (head, position chunk)                              (items split over CTAs)
@@ -14,10 +13,19 @@
 // a per-CTA argmax. The residual stream x is held, identically, in every
 // CTA's shared memory: each CTA adds the same values in the same order.
 //
+// Exchange between phases: every value a phase publishes is one 64-bit word,
+// (epoch tag << 32) | float bits, stored once. A reader polls the words it
+// needs until each carries the epoch of the current (step, layer, phase); the
+// wait and the read are the same L2 round trip, and no grid-wide barrier is
+// needed. A buffer is rewritten only one layer later, after an exchange that
+// every reader of the old contents had to join first, so no reader can miss
+// its data (the per-step argmax candidates, which can lack such an exchange
+// when there are no layers, are double-buffered by step parity).
+//
 // Weights never depend on activations, so the producer warp of each CTA
 // streams its rows of every phase, in order, through the stage ring without
-// waiting for the barriers: while the consumers wait at a barrier, the next
-// phases' weights are already landing. HBM stays busy across the barriers.
+// waiting for the exchanges: while consumers wait on one, the next phases'
+// weights are already landing. HBM stays busy across the waits.
 #pragma once
 #include "stream_gemv.cuh"
 
@@ -25,6 +33,7 @@ namespace tvl {
 
 constexpr int kAttMinChunk = 32;    // positions per attention work item, at least
 constexpr int kAttMaxChunk = 1024;  // and at most
+constexpr int kPhasesPerLayer = 5;  // exchanges per layer: qkv, att, o, h13, f
 
 struct DecodeArgs {
   // weights (inside the arena)
@@ -37,18 +46,16 @@ struct DecodeArgs {
   const float2* rope;  // [S][hd/2] (cos, sin)
   float* kc;           // [L][S][kvd]
   float* vc;
-  // scratch
-  float* qkv;     // [d + 2 kvd]
-  float* o_out;   // [d]
-  float* h13;     // [2F]
-  float* f_out;   // [d]
-  float* logits;  // [V]
-  float* att;     // [H][nch_cap][att_stride]: m, l, -, -, o[hd]
-  float* cand_val;
-  int* cand_idx;  // [G]
-  int* tokens;    // [S]
-  unsigned long long* ts;   // [S]
-  unsigned long long* bar;  // grid barrier counter (monotonic)
+  // tagged exchange buffers (64-bit words: tag << 32 | float bits)
+  unsigned long long* x_qkv;   // [d + 2 kvd]
+  unsigned long long* x_att;   // [H][nch_cap][att_stride]: m, l, -, -, o[hd]
+  unsigned long long* x_o;     // [d]
+  unsigned long long* x_h13;   // [2F]
+  unsigned long long* x_f;     // [d]
+  unsigned long long* x_cand;  // [2][G][2]: per step parity, per CTA (value, index)
+  float* logits;               // [V]
+  int* tokens;                 // [S]
+  unsigned long long* ts;      // [S]
   int* err;
   int* err_host;  // mapped pinned host word (may be null)
   // shape
@@ -57,9 +64,10 @@ struct DecodeArgs {
   float eps, att_scale;
   // this launch
   int start_token, start_pos, n_steps, final_token;
+  unsigned epoch0;  // tag of the first exchange of this launch
   int nst;
   int sm_ring, sm_bars, sm_xs, sm_vec, sm_pdot, sm_att, sm_misc;  // byte offsets
-  unsigned long long barrier_limit_ns;
+  unsigned long long wait_limit_ns;
 };
 
 __host__ __device__ inline int ceil_div_i(int a, int b) { return (a + b - 1) / b; }
@@ -77,54 +85,153 @@ __host__ __device__ inline void att_split(int pos, int H, int G, int* nch, int* 
   *nch = ceil_div_i(n, *clen);
 }
 
-// ---- grid barrier ------------------------------------------------------------
+// ---- tagged exchange -------------------------------------------------------------
 
-// Thread 0 of each CTA arrives on a monotonic 64-bit counter and spins until
-// it reaches base + n*G. The spin is bounded in time; on expiry the kernel
-// raises TVL_E_TIMEOUT and every CTA leaves at its next barrier or wait.
-struct GridBar {
-  unsigned long long base = 0, n = 0;
+__device__ __forceinline__ void st_tag(unsigned long long* p, unsigned tag, float v) {
+  const unsigned long long w =
+      ((unsigned long long)tag << 32) | (unsigned long long)__float_as_uint(v);
+  asm volatile("st.global.cg.u64 [%0], %1;" ::"l"(p), "l"(w) : "memory");
+}
 
-  __device__ void init(const DecodeArgs& a) {
-    if (threadIdx.x == 0) {
-      // No CTA of this launch can pass the first barrier before this one
-      // arrives, so the counter holds k*G + (arrivals so far < G).
-      const unsigned long long v = ld_acquire_u64(a.bar);
-      base = v - v % (unsigned long long)a.G;
+__device__ __forceinline__ ulonglong2 ld_tag2(const unsigned long long* p) {
+  ulonglong2 v;
+  asm volatile("ld.global.cg.v2.u64 {%0, %1}, [%2];" : "=l"(v.x), "=l"(v.y) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ bool tags_are(const ulonglong2& v, unsigned tag) {
+  return (unsigned)(v.x >> 32) == tag && (unsigned)(v.y >> 32) == tag;
+}
+
+__device__ __forceinline__ float lo_f(unsigned long long w) { return __uint_as_float((unsigned)w); }
+
+struct Poll {
+  int* err;
+  int* err_host;
+  volatile int* s_abort;
+  unsigned long long limit_ns;
+};
+
+// Bounded-wait bookkeeping of one polling thread: gives up on abort, on an
+// error raised elsewhere, or after the limit (raising TVL_E_TIMEOUT).
+struct PollClock {
+  uint64_t t0 = 0;
+  uint32_t it = 0;
+  __device__ __forceinline__ bool keep_waiting(const Poll& c) {
+    if ((++it & 15u) != 0) return true;
+    if (*c.s_abort || ld_volatile_s32(c.err)) return false;
+    const uint64_t now = globaltimer_ns();
+    if (t0 == 0) t0 = now;
+    if (now - t0 > c.limit_ns || it > (1u << 24)) {
+      raise_error(c.err, c.err_host, kErrTimeout);
+      *c.s_abort = 1;
+      return false;
     }
+    return true;
   }
+};
 
-  __device__ bool sync(const DecodeArgs& a, volatile int* s_abort) {
-    named_bar_sync(kBarConsumers, kConsumerThreads);
-    bool give_up = false;
-    if (threadIdx.x == 0) {
-      n += 1;
-      const unsigned long long target = base + n * (unsigned long long)a.G;
-      __threadfence();
-      red_release_add_u64(a.bar, 1ull);
-      if (!*s_abort) {
-        const uint64_t t0 = globaltimer_ns();
-        for (uint32_t it = 0;; ++it) {
-          if (ld_acquire_u64(a.bar) >= target) break;
-          if ((it & 31u) == 31u) {
-            if (ld_volatile_s32(a.err)) {
-              *s_abort = 1;
-              break;
-            }
-            if (globaltimer_ns() - t0 > a.barrier_limit_ns || it > (1u << 22)) {
-              raise_error(a.err, a.err_host, kErrTimeout);
-              *s_abort = 1;
-              break;
-            }
+// Poll pairs p = tid, tid + 256, ... of a tagged vector (npairs pairs), up to
+// four 16-byte loads in flight per thread; every not-yet-current pair of a
+// batch is re-read together, so waiting costs one round trip after the last
+// producer's store. fn(p, v0, v1) takes each ready pair. Returns false if this
+// thread gave up (the caller votes).
+template <class Fn>
+__device__ inline bool poll_pairs(const unsigned long long* src, int npairs, unsigned tag,
+                                  const Poll& c, Fn fn) {
+  for (int base = threadIdx.x; base < npairs; base += kConsumerThreads * 4) {
+    ulonglong2 v[4];
+    unsigned pending = 0;
+#pragma unroll
+    for (int b = 0; b < 4; ++b) {
+      const int p = base + b * kConsumerThreads;
+      if (p < npairs) {
+        v[b] = ld_tag2(src + 2 * p);
+        pending |= 1u << b;
+      }
+    }
+    PollClock clk;
+    while (true) {
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        if ((pending >> b) & 1u) {
+          if (tags_are(v[b], tag)) {
+            fn(base + b * kConsumerThreads, lo_f(v[b].x), lo_f(v[b].y));
+            pending &= ~(1u << b);
           }
         }
       }
-      give_up = *s_abort != 0;
+      if (!pending) break;
+      if (!clk.keep_waiting(c)) return false;
+#pragma unroll
+      for (int b = 0; b < 4; ++b)
+        if ((pending >> b) & 1u) v[b] = ld_tag2(src + 2 * (base + b * kConsumerThreads));
     }
-    // thread 0's verdict, given to every consumer thread by a barrier vote
-    return !named_bar_or(kBarConsumers, kConsumerThreads, give_up);
   }
-};
+  return true;
+}
+
+// Same, over two tagged vectors read in step: fn(p, a0, a1, b0, b1).
+template <class Fn>
+__device__ inline bool poll_pairs2(const unsigned long long* sa, const unsigned long long* sb,
+                                   int npairs, unsigned tag, const Poll& c, Fn fn) {
+  for (int base = threadIdx.x; base < npairs; base += kConsumerThreads * 4) {
+    ulonglong2 va[4], vb[4];
+    unsigned pending = 0;
+#pragma unroll
+    for (int b = 0; b < 4; ++b) {
+      const int p = base + b * kConsumerThreads;
+      if (p < npairs) {
+        va[b] = ld_tag2(sa + 2 * p);
+        vb[b] = ld_tag2(sb + 2 * p);
+        pending |= 1u << b;
+      }
+    }
+    PollClock clk;
+    while (true) {
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        if (((pending >> b) & 1u) && tags_are(va[b], tag) && tags_are(vb[b], tag)) {
+          fn(base + b * kConsumerThreads, lo_f(va[b].x), lo_f(va[b].y), lo_f(vb[b].x),
+             lo_f(vb[b].y));
+          pending &= ~(1u << b);
+        }
+      }
+      if (!pending) break;
+      if (!clk.keep_waiting(c)) return false;
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        if ((pending >> b) & 1u) {
+          const int p = base + b * kConsumerThreads;
+          va[b] = ld_tag2(sa + 2 * p);
+          vb[b] = ld_tag2(sb + 2 * p);
+        }
+      }
+    }
+  }
+  return true;
+}
+
+// One pair, re-read until current (used where a thread needs a single pair).
+__device__ inline bool poll_one(const unsigned long long* p, unsigned tag, const Poll& c,
+                                ulonglong2& v) {
+  v = ld_tag2(p);
+  PollClock clk;
+  while (!tags_are(v, tag)) {
+    if (!clk.keep_waiting(c)) return false;
+    v = ld_tag2(p);
+  }
+  return true;
+}
+
+// Leaves the consumer warps together if any of them gave up.
+__device__ __forceinline__ bool vote_ok(bool ok, volatile int* s_abort) {
+  if (named_bar_or(kBarConsumers, kConsumerThreads, !ok)) {
+    if (threadIdx.x == 0) *s_abort = 1;
+    return false;
+  }
+  return true;
+}
 
 // ---- small block-level pieces (consumer threads only) --------------------------
 
@@ -175,30 +282,44 @@ __device__ inline void block_argmax(float& v, int& idx, float* redv, int* redi) 
   named_bar_sync(kBarConsumers, kConsumerThreads);
 }
 
-// out = RMSNorm(x, g) (paper §11.2: ss/n + eps, 1/sqrt, then (x*g)*r).
+// out = RMSNorm(x, g) (paper §11.2: ss/n + eps, 1/sqrt, then (x*g)*r). The
+// gain loads are issued before the reduction so that their latency overlaps it.
 __device__ inline void rmsnorm_to(float* out, const float* x, const float* g, int n, float eps,
                                   float* red) {
+  const int n4 = n >> 2;
+  const float4* g4 = reinterpret_cast<const float4*>(g);
+  float4 gp[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int j = threadIdx.x + k * kConsumerThreads;
+    if (j < n4) gp[k] = __ldg(g4 + j);
+  }
   float ss = 0.f;
   for (int j = threadIdx.x; j < n; j += kConsumerThreads) ss = fmaf(x[j], x[j], ss);
   const float tot = block_sum(ss, red);
   const float r = 1.0f / sqrtf(tot / (float)n + eps);
-  for (int j = threadIdx.x; j < n; j += kConsumerThreads) out[j] = (x[j] * __ldg(g + j)) * r;
-  named_bar_sync(kBarConsumers, kConsumerThreads);
-}
-
-__device__ inline void residual_add(float* x, const float* y, int n) {
-  for (int j = threadIdx.x; j < n; j += kConsumerThreads) x[j] += ldcg(y + j);
-  named_bar_sync(kBarConsumers, kConsumerThreads);
-}
-
-// h = silu(W1 x_b) * (W3 x_b) (paper §2.1, SwiGLU).
-__device__ inline void swiglu_to(float* h, const float* ab, int F) {
-  for (int k = threadIdx.x; k < F; k += kConsumerThreads) {
-    const float a = ldcg(ab + k), b = ldcg(ab + F + k);
-    h[k] = (a / (1.0f + expf(-a))) * b;
+  const float4* x4 = reinterpret_cast<const float4*>(x);
+  float4* o4 = reinterpret_cast<float4*>(out);
+  auto emit = [&](int j, const float4& gv) {
+    const float4 xv = x4[j];
+    o4[j] = make_float4((xv.x * gv.x) * r, (xv.y * gv.y) * r, (xv.z * gv.z) * r,
+                        (xv.w * gv.w) * r);
+  };
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int j = threadIdx.x + k * kConsumerThreads;
+    if (j < n4) emit(j, gp[k]);
   }
+  for (int j = threadIdx.x + 4 * kConsumerThreads; j < n4; j += kConsumerThreads)
+    emit(j, __ldg(g4 + j));
   named_bar_sync(kBarConsumers, kConsumerThreads);
 }
+
+struct EpiTag {
+  unsigned long long* out;
+  unsigned tag;
+  __device__ __forceinline__ void store(int row, float v) { st_tag(out + row, tag, v); }
+};
 
 struct EpiArgmax {
   float* out;
@@ -213,9 +334,10 @@ struct EpiArgmax {
 // ---- attention -------------------------------------------------------------------
 
 // Attention partials of this CTA's items for layer l at position pos. Item
-// (h, c): query head h over the positions of chunk c; writes the chunk's
+// (h, c): query head h over the positions of chunk c; publishes the chunk's
 // max score m, sum of exp(s - m), and sum of exp(s - m) * v.
-__device__ inline void attention_phase(const DecodeArgs& a, int l, int pos, float* sm, float* red) {
+__device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsigned tag_qkv,
+                                       unsigned tag_att, float* sm, float* red, const Poll& pc) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int hd = a.hd, hd4 = hd >> 2, half = hd >> 1;
   int nch, clen;
@@ -240,23 +362,29 @@ __device__ inline void attention_phase(const DecodeArgs& a, int l, int pos, floa
     const int t0 = c * clen;
     const int t1 = (t0 + clen < pos + 1) ? t0 + clen : pos + 1;
     const bool has_new = (t1 == pos + 1);
-    // q (and the new k, v) with RoPE: pair i turns by pos * theta^(-2i/hd)
-    for (int i = tid; i < half; i += kConsumerThreads) {
-      const float2 cs = rp[i];
-      const float qa = ldcg(a.qkv + h * hd + 2 * i), qb = ldcg(a.qkv + h * hd + 2 * i + 1);
-      q[2 * i] = qa * cs.x - qb * cs.y;
-      q[2 * i + 1] = qa * cs.y + qb * cs.x;
-      if (has_new) {
-        const float* kk = a.qkv + a.d + kvh * hd;
-        const float ka = ldcg(kk + 2 * i), kb = ldcg(kk + 2 * i + 1);
-        kp[2 * i] = ka * cs.x - kb * cs.y;
-        kp[2 * i + 1] = ka * cs.y + kb * cs.x;
-        const float* vv = a.qkv + a.d + a.kvd + kvh * hd;
-        vp[2 * i] = ldcg(vv + 2 * i);
-        vp[2 * i + 1] = ldcg(vv + 2 * i + 1);
+    // q (and the new k, v) with RoPE: pair i turns by pos * theta^(-2i/hd).
+    // Pair i of a head is one 16-byte tagged load.
+    const int nget = has_new ? 3 * half : half;
+    bool ok = true;
+    for (int t = tid; t < nget && ok; t += kConsumerThreads) {
+      const int which = t / half, i = t - which * half;
+      const unsigned long long* src =
+          a.x_qkv + (which == 0 ? h * hd : a.d + (which - 1) * a.kvd + kvh * hd) + 2 * i;
+      ulonglong2 v;
+      ok = poll_one(src, tag_qkv, pc, v);
+      const float x0 = lo_f(v.x), x1 = lo_f(v.y);
+      if (which == 2) {
+        vp[2 * i] = x0;
+        vp[2 * i + 1] = x1;
+      } else {
+        const float2 cs = rp[i];
+        float* dst = which == 0 ? q : kp;
+        dst[2 * i] = x0 * cs.x - x1 * cs.y;
+        dst[2 * i + 1] = x0 * cs.y + x1 * cs.x;
       }
     }
-    named_bar_sync(kBarConsumers, kConsumerThreads);
+    if (!vote_ok(ok, pc.s_abort)) return false;
+    __threadfence();  // the K/V rows below were published by other CTAs' earlier steps
     if (has_new && (h % group) == 0) {  // one writer per kv head
       float* kd = a.kc + lay + (size_t)pos * a.kvd + kvh * hd;
       float* vd = a.vc + lay + (size_t)pos * a.kvd + kvh * hd;
@@ -264,31 +392,52 @@ __device__ inline void attention_phase(const DecodeArgs& a, int l, int pos, floa
         kd[j] = kp[j];
         vd[j] = vp[j];
       }
+      __threadfence();  // cache row visible before this item's partials are
     }
-    // scores s_t = (q . k_t) * scale for t in [t0, t1)
+    // scores s_t = (q . k_t) * scale for t in [t0, t1), two passes of loads in flight
     const float4* q4 = reinterpret_cast<const float4*>(q);
-    for (int tb = t0 + warp * ppw; tb < t1; tb += kConsumerWarps * ppw) {
-      const int t = tb + sub;
-      float acc = 0.f;
-      if (t < t1) {
-        const float4* k4 = (t == pos)
-                               ? reinterpret_cast<const float4*>(kp)
-                               : reinterpret_cast<const float4*>(a.kc + lay + (size_t)t * a.kvd +
-                                                                 kvh * hd);
-        for (int f = li; f < hd4; f += lpp) {
-          const float4 kv = (t == pos) ? k4[f] : ldcg4(k4 + f);
-          const float4 qv = q4[f];
-          acc = fmaf(qv.x, kv.x, acc);
-          acc = fmaf(qv.y, kv.y, acc);
-          acc = fmaf(qv.z, kv.z, acc);
-          acc = fmaf(qv.w, kv.w, acc);
+    const int pstride = kConsumerWarps * ppw;
+    for (int tb = t0 + warp * ppw; tb < t1; tb += 2 * pstride) {
+      float acc[2] = {0.f, 0.f};
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int t = tb + u * pstride + sub;
+        if (t < t1) {
+          const float4* k4 = (t == pos)
+                                 ? reinterpret_cast<const float4*>(kp)
+                                 : reinterpret_cast<const float4*>(a.kc + lay + (size_t)t * a.kvd +
+                                                                   kvh * hd);
+          for (int f = li; f < hd4; f += lpp) {
+            const float4 kv = (t == pos) ? k4[f] : ldcg4(k4 + f);
+            const float4 qv = q4[f];
+            acc[u] = fmaf(qv.x, kv.x, acc[u]);
+            acc[u] = fmaf(qv.y, kv.y, acc[u]);
+            acc[u] = fmaf(qv.z, kv.z, acc[u]);
+            acc[u] = fmaf(qv.w, kv.w, acc[u]);
+          }
         }
       }
-      for (int o = lpp >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-      if (t < t1 && li == 0) sc[t - t0] = acc * a.att_scale;
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int t = tb + u * pstride + sub;
+        float s = acc[u];
+        for (int o = lpp >> 1; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if (t < t1 && li == 0) sc[t - t0] = s * a.att_scale;
+      }
     }
-    named_bar_sync(kBarConsumers, kConsumerThreads);
+    // V rows of the first positions of this thread, loaded while the softmax runs
+    const int ng = kConsumerThreads / hd4;
+    const int gi = tid / hd4, f = tid - gi * hd4;
     const int n = t1 - t0;
+    auto vrow = [&](int t) -> float4 {
+      return (t == pos) ? reinterpret_cast<const float4*>(vp)[f]
+                        : ldcg4(reinterpret_cast<const float4*>(a.vc + lay + (size_t)t * a.kvd +
+                                                                kvh * hd) + f);
+    };
+    float4 v0 = make_float4(0.f, 0.f, 0.f, 0.f), v1 = v0;
+    if (gi < ng && gi < n) v0 = vrow(t0 + gi);
+    if (gi < ng && gi + ng < n) v1 = vrow(t0 + gi + ng);
+    named_bar_sync(kBarConsumers, kConsumerThreads);
     float m = -INFINITY;
     for (int i = tid; i < n; i += kConsumerThreads) m = fmaxf(m, sc[i]);
     m = block_max(m, red);
@@ -299,54 +448,55 @@ __device__ inline void attention_phase(const DecodeArgs& a, int l, int pos, floa
       ls += e;
     }
     ls = block_sum(ls, red);  // its barriers also publish sc
-    // o = sum_t e_t v_t: thread (g, f) sums float4 column f over t = g, g+ng, ...
-    const int ng = kConsumerThreads / hd4;
-    const int gi = tid / hd4, f = tid - gi * hd4;
+    // o = sum_t e_t v_t: thread (gi, f) sums float4 column f over t = gi, gi+ng, ...
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     if (gi < ng) {
-      for (int i = gi; i < n; i += ng) {
-        const int t = t0 + i;
-        const float e = sc[i];
-        const float4 vv =
-            (t == pos) ? reinterpret_cast<const float4*>(vp)[f]
-                       : ldcg4(reinterpret_cast<const float4*>(a.vc + lay + (size_t)t * a.kvd +
-                                                               kvh * hd) + f);
+      auto fma4 = [&](float e, const float4& vv) {
         acc.x = fmaf(e, vv.x, acc.x);
         acc.y = fmaf(e, vv.y, acc.y);
         acc.z = fmaf(e, vv.z, acc.z);
         acc.w = fmaf(e, vv.w, acc.w);
-      }
+      };
+      if (gi < n) fma4(sc[gi], v0);
+      if (gi + ng < n) fma4(sc[gi + ng], v1);
+      for (int i = gi + 2 * ng; i < n; i += ng) fma4(sc[i], vrow(t0 + i));
       reinterpret_cast<float4*>(part)[gi * hd4 + f] = acc;
     }
     named_bar_sync(kBarConsumers, kConsumerThreads);
-    float* rec = a.att + ((size_t)h * a.nch_cap + c) * a.att_stride;
+    unsigned long long* rec = a.x_att + ((size_t)h * a.nch_cap + c) * a.att_stride;
     for (int j = tid; j < hd; j += kConsumerThreads) {
       float o = 0.f;
       for (int g2 = 0; g2 < ng; ++g2) o += part[g2 * hd + j];
-      rec[4 + j] = o;
+      st_tag(rec + 4 + j, tag_att, o);
     }
     if (tid == 0) {
-      rec[0] = m;
-      rec[1] = ls;
+      st_tag(rec, tag_att, m);
+      st_tag(rec + 1, tag_att, ls);
     }
     named_bar_sync(kBarConsumers, kConsumerThreads);
   }
+  return true;
 }
 
-// o[h*hd + j] = sum_c w_c o_c[j] / sum_c w_c l_c with w_c = exp(m_c - max m).
-__device__ inline void merge_attention(const DecodeArgs& a, int pos, float* o, float* sm) {
+// o[h*hd + j] = sum_c w_c o_c[j] with w_c = exp(m_c - M) / sum_c exp(m_c - M) l_c.
+__device__ inline bool merge_attention(const DecodeArgs& a, int pos, unsigned tag, float* o,
+                                       float* sm, const Poll& pc) {
   const int tid = threadIdx.x;
   int nch, clen;
   att_split(pos, a.H, a.G, &nch, &clen);
   const int nrec = a.H * nch;
   float* mv = sm;         // [H * nch]
   float* wv = sm + nrec;  // [H * nch]
-  for (int i = tid; i < nrec; i += kConsumerThreads) {
+  bool ok = true;
+  for (int i = tid; i < nrec && ok; i += kConsumerThreads) {
     const int h = i / nch, c = i - h * nch;
-    mv[i] = ldcg(a.att + ((size_t)h * a.nch_cap + c) * a.att_stride);
-    wv[i] = ldcg(a.att + ((size_t)h * a.nch_cap + c) * a.att_stride + 1);
+    const unsigned long long* src = a.x_att + ((size_t)h * a.nch_cap + c) * a.att_stride;
+    ulonglong2 v;
+    ok = poll_one(src, tag, pc, v);
+    mv[i] = lo_f(v.x);
+    wv[i] = lo_f(v.y);
   }
-  named_bar_sync(kBarConsumers, kConsumerThreads);
+  if (!vote_ok(ok, pc.s_abort)) return false;
   for (int h = tid; h < a.H; h += kConsumerThreads) {
     float M = -INFINITY;
     for (int c = 0; c < nch; ++c) M = fmaxf(M, mv[h * nch + c]);
@@ -355,58 +505,109 @@ __device__ inline void merge_attention(const DecodeArgs& a, int pos, float* o, f
     for (int c = 0; c < nch; ++c) wv[h * nch + c] = expf(mv[h * nch + c] - M) / Lsum;
   }
   named_bar_sync(kBarConsumers, kConsumerThreads);
-  for (int e = tid; e < a.d; e += kConsumerThreads) {
-    const int h = e / a.hd, j = e - h * a.hd;
-    float acc = 0.f;
-    for (int c = 0; c < nch; ++c)
-      acc = fmaf(wv[h * nch + c], ldcg(a.att + ((size_t)h * a.nch_cap + c) * a.att_stride + 4 + j),
-                 acc);
-    o[e] = acc;
+  // output pairs (2p, 2p+1) of head h = 2p / hd: one 16-byte load per chunk,
+  // up to eight chunks in flight, re-read together until current
+  const int half = a.hd >> 1;
+  for (int p = tid; p < (a.d >> 1) && ok; p += kConsumerThreads) {
+    const int h = p / half, jp = p - h * half;
+    const unsigned long long* rec0 = a.x_att + (size_t)h * a.nch_cap * a.att_stride + 4 + 2 * jp;
+    float s0 = 0.f, s1 = 0.f;
+    for (int cb = 0; cb < nch && ok; cb += 8) {
+      const int ce = (nch - cb < 8) ? nch - cb : 8;
+      ulonglong2 v[8];
+      unsigned pending = 0;
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+        if (k < ce) {
+          v[k] = ld_tag2(rec0 + (size_t)(cb + k) * a.att_stride);
+          pending |= 1u << k;
+        }
+      PollClock clk;
+      while (ok) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          if (((pending >> k) & 1u) && tags_are(v[k], tag)) pending &= ~(1u << k);
+        if (!pending) break;
+        ok = clk.keep_waiting(pc);
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          if ((pending >> k) & 1u) v[k] = ld_tag2(rec0 + (size_t)(cb + k) * a.att_stride);
+      }
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        if (k < ce) {  // chunk order: the same sum in every CTA
+          const float w = wv[h * nch + cb + k];
+          s0 = fmaf(w, lo_f(v[k].x), s0);
+          s1 = fmaf(w, lo_f(v[k].y), s1);
+        }
+      }
+    }
+    o[2 * p] = s0;
+    o[2 * p + 1] = s1;
   }
-  named_bar_sync(kBarConsumers, kConsumerThreads);
+  return vote_ok(ok, pc.s_abort);
 }
 
 // Next token: argmax over the per-CTA candidates (identical in every CTA).
-__device__ inline int reduce_candidates(const DecodeArgs& a, float* redv, int* redi) {
+__device__ inline bool reduce_candidates(const DecodeArgs& a, int parity, unsigned tag,
+                                         float* redv, int* redi, const Poll& pc, int* token) {
   float bv = -INFINITY;
   int bi = 0x7fffffff;
-  for (int c = threadIdx.x; c < a.G; c += kConsumerThreads) {
-    const float v = ldcg(a.cand_val + c);
-    const int i = __ldcg(a.cand_idx + c);
+  const unsigned long long* base = a.x_cand + (size_t)parity * a.G * 2;
+  const bool ok = poll_pairs(base, a.G, tag, pc, [&](int p, float v, float idx) {
+    const int i = (int)__float_as_uint(idx);
     if (better(v, i, bv, bi)) { bv = v; bi = i; }
-  }
+  });
+  if (!vote_ok(ok, pc.s_abort)) return false;
   block_argmax(bv, bi, redv, redi);
-  return bi;
+  *token = (bi >= 0 && bi < a.V) ? bi : 0;  // 0 only if every logit was NaN
+  return true;
 }
 
 // ---- the kernel --------------------------------------------------------------------
 
-__device__ inline void decode_producer(const DecodeArgs& a, const Ring& r, volatile int* s_abort) {
-  const uint64_t pol = l2_evict_first();
-  const int c = blockIdx.x;
-  uint32_t g = 0;
-  bool ok = true;
-  for (int s = 0; s < a.n_steps && ok; ++s) {
-    for (int l = 0; l < a.L && ok; ++l) {
-      const unsigned char* lw = a.layer0 + (size_t)l * a.layer_stride;
-      ok = produce_phase(r, g, reinterpret_cast<const float*>(lw + a.o_wqkv),
-                         plan_stages(a.d + 2 * a.kvd, a.d, a.G, c), pol, a.err, a.err_host,
-                         s_abort) &&
-           produce_phase(r, g, reinterpret_cast<const float*>(lw + a.o_wo),
-                         plan_stages(a.d, a.d, a.G, c), pol, a.err, a.err_host, s_abort) &&
-           produce_phase(r, g, reinterpret_cast<const float*>(lw + a.o_w13),
-                         plan_stages(2 * a.F, a.d, a.G, c), pol, a.err, a.err_host, s_abort) &&
-           produce_phase(r, g, reinterpret_cast<const float*>(lw + a.o_w2),
-                         plan_stages(a.d, a.F, a.G, c), pol, a.err, a.err_host, s_abort);
+// The weight stream of one launch, in consumption order: per step, each
+// layer's [Wq|Wk|Wv], Wo, [W1|W3], W2, then the classifier; this CTA's rows.
+struct DecodeSched {
+  const DecodeArgs* a;
+  int s = 0, l = 0, k = 0;
+  __device__ bool next(const float*& W, StagePlan& p) {
+    if (s >= a->n_steps) return false;
+    const int c = blockIdx.x;
+    if (l < a->L) {
+      const unsigned char* lw = a->layer0 + (size_t)l * a->layer_stride;
+      if (k == 0) {
+        W = reinterpret_cast<const float*>(lw + a->o_wqkv);
+        p = plan_stages(a->d + 2 * a->kvd, a->d, a->G, c);
+      } else if (k == 1) {
+        W = reinterpret_cast<const float*>(lw + a->o_wo);
+        p = plan_stages(a->d, a->d, a->G, c);
+      } else if (k == 2) {
+        W = reinterpret_cast<const float*>(lw + a->o_w13);
+        p = plan_stages(2 * a->F, a->d, a->G, c);
+      } else {
+        W = reinterpret_cast<const float*>(lw + a->o_w2);
+        p = plan_stages(a->d, a->F, a->G, c);
+      }
+      if (++k == 4) {
+        k = 0;
+        ++l;
+      }
+      return true;
     }
-    ok = ok && produce_phase(r, g, a.Wcls, plan_stages(a.V, a.d, a.G, c), pol, a.err, a.err_host,
-                             s_abort);
+    W = a->Wcls;
+    p = plan_stages(a->V, a->d, a->G, c);
+    l = 0;
+    k = 0;
+    ++s;
+    return true;
   }
-  drain_ring(r, g);
-}
+};
 
-__device__ inline void decode_consumer(const DecodeArgs& a, const Ring& r, unsigned char* smem,
-                                       volatile int* s_abort) {
+using DecodeFeeder = Feeder<DecodeSched>;
+
+__device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, DecodeFeeder& feed,
+                                    uint32_t& g, unsigned char* smem, volatile int* s_abort) {
   float* xs = reinterpret_cast<float*>(smem + a.sm_xs);
   float* vec = reinterpret_cast<float*>(smem + a.sm_vec);
   float* pdot = reinterpret_cast<float*>(smem + a.sm_pdot);
@@ -414,15 +615,22 @@ __device__ inline void decode_consumer(const DecodeArgs& a, const Ring& r, unsig
   float* red = reinterpret_cast<float*>(smem + a.sm_misc) + 8;
   int* redi = reinterpret_cast<int*>(smem + a.sm_misc) + 24;
   const int tid = threadIdx.x, c = blockIdx.x;
-  uint32_t g = 0;
-  GridBar gb;
-  gb.init(a);
+  const Poll pc{a.err, a.err_host, s_abort, a.wait_limit_ns};
+  const unsigned per_step = (unsigned)(kPhasesPerLayer * a.L + 1);
   int token = a.start_token;
+  // x += (published vector), identically in every CTA
+  auto add_published = [&](const unsigned long long* src, unsigned tag) {
+    const bool ok = poll_pairs(src, a.d >> 1, tag, pc, [&](int p, float v0, float v1) {
+      xs[2 * p] += v0;
+      xs[2 * p + 1] += v1;
+    });
+    return vote_ok(ok, s_abort);
+  };
   for (int s = 0; s < a.n_steps; ++s) {
     const int pos = a.start_pos + s;
+    const unsigned es = a.epoch0 + (unsigned)s * per_step;
     if (s > 0) {
-      token = reduce_candidates(a, red, redi);
-      if (token < 0 || token >= a.V) token = 0;  // only if every logit was NaN
+      if (!reduce_candidates(a, (s - 1) & 1, es - 1, red, redi, pc, &token)) return false;
       if (c == 0 && tid == 0) {
         a.tokens[s - 1] = token;
         a.ts[s - 1] = globaltimer_ns();
@@ -435,94 +643,98 @@ __device__ inline void decode_consumer(const DecodeArgs& a, const Ring& r, unsig
     named_bar_sync(kBarConsumers, kConsumerThreads);
     for (int l = 0; l < a.L; ++l) {
       const unsigned char* lw = a.layer0 + (size_t)l * a.layer_stride;
+      const unsigned el = es + (unsigned)(kPhasesPerLayer * l);
+      if (l > 0 && !add_published(a.x_f, el - 1)) return false;
       rmsnorm_to(vec, xs, reinterpret_cast<const float*>(lw + a.o_gatt), a.d, a.eps, red);
-      EpiStore e_qkv{a.qkv};
-      if (!consume_phase(r, g, plan_stages(a.d + 2 * a.kvd, a.d, a.G, c), vec, 1, a.d, pdot,
+      EpiTag e_qkv{a.x_qkv, el};
+      if (!consume_phase(r, g, feed, plan_stages(a.d + 2 * a.kvd, a.d, a.G, c), vec, 1, a.d, pdot,
                          e_qkv, a.err, a.err_host, s_abort))
-        return;
-      if (!gb.sync(a, s_abort)) return;
-      attention_phase(a, l, pos, asm_, red);
-      if (!gb.sync(a, s_abort)) return;
-      merge_attention(a, pos, vec, asm_);
-      EpiStore e_o{a.o_out};
-      if (!consume_phase(r, g, plan_stages(a.d, a.d, a.G, c), vec, 1, a.d, pdot, e_o, a.err,
+        return false;
+      if (!attention_phase(a, l, pos, el, el + 1, asm_, red, pc)) return false;
+      if (!merge_attention(a, pos, el + 1, vec, asm_, pc)) return false;
+      EpiTag e_o{a.x_o, el + 2};
+      if (!consume_phase(r, g, feed, plan_stages(a.d, a.d, a.G, c), vec, 1, a.d, pdot, e_o, a.err,
                          a.err_host, s_abort))
-        return;
-      if (!gb.sync(a, s_abort)) return;
-      residual_add(xs, a.o_out, a.d);
+        return false;
+      if (!add_published(a.x_o, el + 2)) return false;
       rmsnorm_to(vec, xs, reinterpret_cast<const float*>(lw + a.o_gffn), a.d, a.eps, red);
-      EpiStore e_13{a.h13};
-      if (!consume_phase(r, g, plan_stages(2 * a.F, a.d, a.G, c), vec, 1, a.d, pdot, e_13, a.err,
+      EpiTag e_13{a.x_h13, el + 3};
+      if (!consume_phase(r, g, feed, plan_stages(2 * a.F, a.d, a.G, c), vec, 1, a.d, pdot, e_13, a.err,
                          a.err_host, s_abort))
-        return;
-      if (!gb.sync(a, s_abort)) return;
-      swiglu_to(vec, a.h13, a.F);
-      EpiStore e_2{a.f_out};
-      if (!consume_phase(r, g, plan_stages(a.d, a.F, a.G, c), vec, 1, a.F, pdot, e_2, a.err,
+        return false;
+      {  // h = silu(a) * b (paper §2.1, SwiGLU); a = h13[k], b = h13[F + k]
+        const bool ok = poll_pairs2(a.x_h13, a.x_h13 + a.F, a.F >> 1, el + 3, pc,
+                                    [&](int p, float a0, float a1, float b0, float b1) {
+                                      vec[2 * p] = (a0 / (1.0f + expf(-a0))) * b0;
+                                      vec[2 * p + 1] = (a1 / (1.0f + expf(-a1))) * b1;
+                                    });
+        if (!vote_ok(ok, s_abort)) return false;
+      }
+      EpiTag e_2{a.x_f, el + 4};
+      if (!consume_phase(r, g, feed, plan_stages(a.d, a.F, a.G, c), vec, 1, a.F, pdot, e_2, a.err,
                          a.err_host, s_abort))
-        return;
-      if (!gb.sync(a, s_abort)) return;
-      residual_add(xs, a.f_out, a.d);
+        return false;
     }
+    if (a.L > 0 && !add_published(a.x_f, es + per_step - 2)) return false;
     rmsnorm_to(vec, xs, a.g_final, a.d, a.eps, red);
     EpiArgmax ea{a.logits, -INFINITY, 0x7fffffff};
-    if (!consume_phase(r, g, plan_stages(a.V, a.d, a.G, c), vec, 1, a.d, pdot, ea, a.err,
+    if (!consume_phase(r, g, feed, plan_stages(a.V, a.d, a.G, c), vec, 1, a.d, pdot, ea, a.err,
                        a.err_host, s_abort))
-      return;
+      return false;
     float bv = ea.bv;
     int bi = ea.bi;
     block_argmax(bv, bi, red, redi);
     if (tid == 0) {
-      a.cand_val[c] = bv;
-      a.cand_idx[c] = bi;
-    }
-    if (s + 1 < a.n_steps || a.final_token) {
-      if (!gb.sync(a, s_abort)) return;
+      unsigned long long* dst = a.x_cand + ((size_t)(s & 1) * a.G + c) * 2;
+      st_tag(dst, es + per_step - 1, bv);
+      st_tag(dst + 1, es + per_step - 1, __uint_as_float((unsigned)bi));
     }
   }
   if (a.final_token && c == 0) {
-    token = reduce_candidates(a, red, redi);
+    const int s = a.n_steps - 1;
+    if (!reduce_candidates(a, s & 1, a.epoch0 + (unsigned)a.n_steps * per_step - 1, red, redi,
+                           pc, &token))
+      return false;
     if (tid == 0) {
-      a.tokens[a.n_steps - 1] = token;
-      a.ts[a.n_steps - 1] = globaltimer_ns();
+      a.tokens[s] = token;
+      a.ts[s] = globaltimer_ns();
     }
   }
+  return true;
 }
 
-__global__ void __launch_bounds__(kThreads, 1) decode_kernel(const DecodeArgs a) {
+__global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_constant__ DecodeArgs a) {
   extern __shared__ __align__(128) unsigned char smem[];
   Ring r;
   r.buf = smem + a.sm_ring;
   r.full = reinterpret_cast<uint64_t*>(smem + a.sm_bars);
-  r.empty = r.full + a.nst;
   r.nst = a.nst;
   volatile int* s_abort = reinterpret_cast<volatile int*>(smem + a.sm_misc);
+  __shared__ DecodeFeeder feed;
   if (threadIdx.x == 0) {
-    for (int i = 0; i < a.nst; ++i) {
-      mbar_init(&r.full[i], 1);
-      mbar_init(&r.empty[i], 1);
-    }
+    feed = DecodeFeeder();
+    feed.sched.a = &a;
+    for (int i = 0; i < a.nst; ++i) mbar_init(&r.full[i], 1);
     *s_abort = 0;
     fence_mbar_init();
+    feed.start(r);
   }
   __syncthreads();
-  if (threadIdx.x >= kConsumerThreads) {
-    if (threadIdx.x == kConsumerThreads) decode_producer(a, r, s_abort);
-    return;
-  }
-  decode_consumer(a, r, smem, s_abort);
+  uint32_t g = 0;
+  if (!decode_steps(a, r, feed, g, smem, s_abort) && threadIdx.x == 0) feed.drain(r, g);
 }
 
-// Failure-detection self-test: one barrier whose count nothing will reach.
-__global__ void barrier_selftest_kernel(DecodeArgs a) {
+// Failure-detection self-test: one CTA polls a tagged word that nothing
+// writes; the bounded wait must expire and report TVL_E_TIMEOUT.
+__global__ void wait_selftest_kernel(unsigned long long* word, int* err,
+                                     unsigned long long limit_ns) {
   __shared__ int s_abort;
   if (threadIdx.x == 0) s_abort = 0;
   __syncthreads();
   if (threadIdx.x >= kConsumerThreads) return;
-  GridBar gb;
-  gb.init(a);
-  if (threadIdx.x == 0) gb.n = 1;  // expect one more full round than will ever arrive
-  gb.sync(a, reinterpret_cast<volatile int*>(&s_abort));
+  const Poll pc{err, nullptr, &s_abort, limit_ns};
+  const bool ok = poll_pairs(word, 1, 1u, pc, [](int, float, float) {});
+  vote_ok(ok, &s_abort);
 }
 
 }  // namespace tvl

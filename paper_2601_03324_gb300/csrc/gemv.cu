@@ -1,7 +1,7 @@
 // gemv.cu — standalone y = W x (paper §6.1) on the weight-streaming engine.
 //
 // One CTA per SM streams its contiguous share of W through the shared-memory
-// stage ring. Matrices with few rows are split along K into S chunks so that
+// stage ring (8 warps; thread 0 keeps the ring full). Matrices with few rows are split along K into S chunks so that
 // every SM gets work: virtual row v = (row v / S, chunk v % S); each virtual
 // row's partial lands in a scratch buffer, and each row is summed over its
 // S chunks in chunk order — by the CTA that owns the whole row, or for a row
@@ -37,32 +37,41 @@ struct EpiPart {
   __device__ __forceinline__ void store(int v, float val) { part[v] = val; }
 };
 
-__global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const GemvArgs a) {
+// The single phase of a standalone GEMV.
+struct GemvSched {
+  const float* W;
+  StagePlan p;
+  bool given;
+  __device__ bool next(const float*& w, StagePlan& plan) {
+    if (given) return false;
+    given = true;
+    w = W;
+    plan = p;
+    return true;
+  }
+};
+
+__global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_constant__ GemvArgs a) {
   extern __shared__ __align__(128) unsigned char smem[];
   Ring r;
   r.buf = smem + a.sm_ring;
   r.full = reinterpret_cast<uint64_t*>(smem + a.sm_bars);
-  r.empty = r.full + a.nst;
   r.nst = a.nst;
   volatile int* s_abort = reinterpret_cast<volatile int*>(smem + a.sm_misc);
+  const StagePlan p = plan_stages(a.nv, a.Kc, gridDim.x, blockIdx.x);
+  __shared__ Feeder<GemvSched> feed;
   if (threadIdx.x == 0) {
-    for (int i = 0; i < a.nst; ++i) {
-      mbar_init(&r.full[i], 1);
-      mbar_init(&r.empty[i], 1);
-    }
+    feed = Feeder<GemvSched>();
+    feed.sched.W = a.W;
+    feed.sched.p = p;
+    feed.sched.given = false;
+    for (int i = 0; i < a.nst; ++i) mbar_init(&r.full[i], 1);
     *s_abort = 0;
     fence_mbar_init();
+    feed.start(r);
   }
   __syncthreads();
-  const StagePlan p = plan_stages(a.nv, a.Kc, gridDim.x, blockIdx.x);
   uint32_t g = 0;
-  if (threadIdx.x >= kConsumerThreads) {
-    if (threadIdx.x == kConsumerThreads) {
-      produce_phase(r, g, a.W, p, l2_evict_first(), nullptr, nullptr, s_abort);
-      drain_ring(r, g);
-    }
-    return;
-  }
   float* xs = reinterpret_cast<float*>(smem + a.sm_x);
   float* pdot = reinterpret_cast<float*>(smem + a.sm_pdot);
   const float4* x4 = reinterpret_cast<const float4*>(a.x);
@@ -71,11 +80,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const GemvArgs
   named_bar_sync(kBarConsumers, kConsumerThreads);
   if (a.S == 1) {
     EpiStore e{a.y};
-    consume_phase(r, g, p, xs, 1, a.Kc, pdot, e, nullptr, nullptr, s_abort);
+    consume_phase(r, g, feed, p, xs, 1, a.Kc, pdot, e, nullptr, nullptr, s_abort);
     return;
   }
   EpiPart e{a.part};
-  if (!consume_phase(r, g, p, xs, a.S, a.Kc, pdot, e, nullptr, nullptr, s_abort)) return;
+  if (!consume_phase(r, g, feed, p, xs, a.S, a.Kc, pdot, e, nullptr, nullptr, s_abort)) return;
   if (p.r1 <= p.r0) return;
   named_bar_sync(kBarConsumers, kConsumerThreads);
   const int S = a.S;
@@ -178,7 +187,8 @@ extern "C" tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t
   const int G = (int)(a.nv < info.sms ? a.nv : info.sms);
   // shared memory: ring | barriers | x | piece sums | misc
   const int xbytes = (int)a128(4LL * d_in), pdot = 2 * kMaxPieces * 4, bars = 128, misc = 128;
-  int nst = (info.max_optin - xbytes - pdot - bars - misc) / kStageBytes;
+  // (minus 1 KB for the kernel's static shared memory)
+  int nst = (info.max_optin - 1024 - xbytes - pdot - bars - misc) / kStageBytes;
   if (nst > 6) nst = 6;
   if (nst < 2) {
     set_error("tvl_gemv: not enough shared memory");

@@ -2,21 +2,23 @@
 // kernel and the standalone GEMV (paper §3.1: y = W x reads every weight once,
 // so the work is bound by memory; §6.1: one dot product per output row).
 //
-// Per CTA: one producer warp streams a contiguous range of weight rows from
-// global memory into a ring of shared-memory stages with bulk asynchronous
-// copies (the TMA engine), each stage completing on an mbarrier; eight
-// consumer warps multiply each landed stage by the input vector held in
-// shared memory. This is the GPU form of the paper's two memory ideas: the
+// Per CTA: a ring of shared-memory stages is filled with bulk asynchronous
+// copies (the TMA engine) of a contiguous range of weight rows, each stage
+// completing on an mbarrier; eight warps multiply each landed stage by the
+// input vector held in shared memory. Thread 0 keeps the ring full: it issues
+// the copy of stage g + nst as soon as stage g is consumed, walking a static
+// schedule of phases that does not depend on activations, so the copies run
+// ahead of whatever the warps are waiting for. This is the GPU form of the paper's two memory ideas: the
 // weights flow as one aligned stream (§3.2, §4.1) and several independent
 // loads are always in flight (§11.1's four accumulators become several
 // 32 KB stages in flight per SM).
 //
 // Work split: CTA c owns rows [M*c/G, M*(c+1)/G) of an [M x K] matrix, which
 // is one contiguous byte range. A stage holds whole rows (when a row fits in
-// a stage) or one segment of a row. Inside a stage, rows are cut into pieces
-// of at most kPiece floats; warps take pieces round-robin, each piece sum is
-// a fixed shuffle tree, and each row sums its pieces in index order, so the
-// result is bit-reproducible.
+// a stage) or one segment of a row. Inside a stage, each row is one unit of
+// work for a warp, or 2/4/8 parts when the stage has fewer rows than warps;
+// each unit sum is a fixed shuffle tree and each row sums its parts in order,
+// so the result is bit-reproducible.
 #pragma once
 #include "ptx.cuh"
 
@@ -24,10 +26,9 @@ namespace tvl {
 
 constexpr int kConsumerWarps = 8;
 constexpr int kConsumerThreads = kConsumerWarps * 32;
-constexpr int kThreads = kConsumerThreads + 32;  // + one producer warp
+constexpr int kThreads = kConsumerThreads;  // 2 warps per SM sub-partition: up to 255 registers
 constexpr int kStageBytes = 32768;
 constexpr int kStageFloats = kStageBytes / 4;
-constexpr int kPiece = 256;           // floats one warp reduces at a time
 constexpr int kMaxRowsPerStage = 256;
 constexpr int kMaxPieces = 256;       // per stage; see plan_stages
 constexpr uint32_t kBarConsumers = 1; // named barrier of the consumer warps
@@ -49,9 +50,9 @@ struct StageDesc {
   int row, nrows, c0, c1;  // rows [row, row+nrows), columns [c0, c1)
 };
 
-// Requires K % 4 == 0 (16-byte rows) and kStageFloats % 32 == 0. Piece bound:
-// K <= kPiece gives one piece per row and at most kMaxRowsPerStage rows;
-// otherwise rows*ceil(K/kPiece) <= kStageFloats/kPiece + kStageFloats/K < 64.
+// Requires K % 4 == 0 (16-byte rows) and kStageFloats % 32 == 0. A stage has
+// at most kMaxRowsPerStage rows; units per stage (rows x parts) stay below
+// max(kMaxRowsPerStage, 2 * kConsumerWarps) <= kMaxPieces.
 __host__ __device__ inline StagePlan plan_stages(long long M, int K, int G, int c) {
   StagePlan p;
   p.r0 = (int)(M * c / G);
@@ -92,8 +93,7 @@ __host__ __device__ inline StageDesc stage_desc(const StagePlan& p, int j) {
 
 struct Ring {
   unsigned char* buf;
-  uint64_t* full;
-  uint64_t* empty;
+  uint64_t* full;  // [nst]
   int nst;
 };
 
@@ -102,7 +102,7 @@ __device__ __forceinline__ void raise_error(int* err, int* err_host, int code) {
   if (err_host) *reinterpret_cast<volatile int*>(err_host) = code;
 }
 
-// Single-thread bounded wait (producer). Gives up on abort, on an error
+// Single-thread bounded wait. Gives up on abort (when honoured), on an error
 // raised elsewhere, or after kWaitLimitNs; returns false then.
 __device__ inline bool wait_bounded(uint64_t* bar, uint32_t par, const int* err,
                                     volatile int* s_abort, bool honour_abort, bool* timed_out) {
@@ -120,42 +120,57 @@ __device__ inline bool wait_bounded(uint64_t* bar, uint32_t par, const int* err,
   }
 }
 
-// Producer: queue the stages of one phase. g counts stages over the launch.
-__device__ inline bool produce_phase(const Ring& r, uint32_t& g, const float* W, const StagePlan& p,
-                                     uint64_t pol, int* err, int* err_host,
-                                     volatile int* s_abort) {
-  for (int j = 0; j < p.nstages; ++j, ++g) {
-    const int slot = (int)(g % (uint32_t)r.nst);
-    if (g >= (uint32_t)r.nst) {
-      bool to = false;
-      const uint32_t par = ((g / (uint32_t)r.nst) - 1u) & 1u;
-      if (!wait_bounded(&r.empty[slot], par, err, s_abort, true, &to)) {
-        if (to) raise_error(err, err_host, kErrTimeout);
-        *s_abort = 1;
-        return false;
+// Queues the stages of a static schedule of GEMV phases into the ring, in
+// order. Sched::next(W, plan) yields the next phase's matrix and this CTA's
+// stage plan, false at the end. Used by thread 0 only; the object lives in
+// shared memory so that its state takes no registers in the stage loop.
+template <class Sched>
+struct Feeder {
+  Sched sched;
+  const float* W = nullptr;
+  StagePlan p{};
+  int j = 0;            // next stage of the current phase
+  uint32_t issued = 0;  // stages queued so far
+  bool done = false;
+  uint64_t pol = 0;
+
+  __device__ void start(const Ring& r) {
+    pol = l2_evict_first();
+    p.nstages = 0;
+    for (int k = 0; k < r.nst; ++k) issue(r);
+  }
+  // Queue the next stage into slot issued % nst (its previous stage has been
+  // consumed: the caller has passed the barrier that ends it).
+  __device__ void issue(const Ring& r) {
+    if (done) return;
+    while (j >= p.nstages) {
+      if (!sched.next(W, p)) {
+        done = true;
+        return;
       }
+      j = 0;
     }
     const StageDesc s = stage_desc(p, j);
     const uint32_t bytes = (uint32_t)(s.nrows * (s.c1 - s.c0)) * 4u;
+    const int slot = (int)(issued % (uint32_t)r.nst);
     mbar_arrive_expect_tx(&r.full[slot], bytes);
     bulk_g2s(r.buf + (size_t)slot * kStageBytes, W + (size_t)s.row * p.K + s.c0, bytes,
              &r.full[slot], pol);
+    ++j;
+    ++issued;
   }
-  return true;
-}
+  // Before the CTA leaves early: wait for the copies still in flight.
+  __device__ void drain(const Ring& r, uint32_t consumed) {
+    for (uint32_t k = consumed; k < issued; ++k)
+      wait_bounded(&r.full[k % (uint32_t)r.nst], (k / (uint32_t)r.nst) & 1u, nullptr, nullptr,
+                   false, nullptr);
+  }
+};
 
-// Producer epilogue: every copy it queued must land before the CTA may exit.
-__device__ inline void drain_ring(const Ring& r, uint32_t g) {
-  const uint32_t from = g > (uint32_t)r.nst ? g - (uint32_t)r.nst : 0u;
-  for (uint32_t k = from; k < g; ++k)
-    wait_bounded(&r.full[k % (uint32_t)r.nst], (k / (uint32_t)r.nst) & 1u, nullptr, nullptr,
-                 false, nullptr);
-}
-
-// All consumer threads poll; thread 0 alone applies the limit and raises
-// the abort flag, which the others observe (the producer may raise it too).
-// Returns true if the stage landed. The flag is only a hint to stop waiting:
-// the decision to leave is taken by a vote at the next barrier.
+// All threads poll; thread 0 alone applies the limit and raises the abort
+// flag, which the others observe. Returns true if the stage landed. The flag
+// is only a hint to stop waiting: the decision to leave is taken by a vote at
+// the next barrier.
 __device__ inline bool consumer_wait_full(uint64_t* bar, uint32_t par, int* err, int* err_host,
                                           volatile int* s_abort) {
   if (mbar_try_wait(bar, par)) return true;
@@ -178,13 +193,47 @@ __device__ inline bool consumer_wait_full(uint64_t* bar, uint32_t par, int* err,
   }
 }
 
+// Lane part of one unit's dot product: n4 <= 256 float4 of weights and
+// input; lane takes float4 lane + 32k (k < 8), in a fully unrolled loop whose
+// loads the compiler hoists as far as registers allow.
+__device__ __forceinline__ float unit_partial(const float4* w4, const float4* x4, int n4,
+                                              int lane) {
+  float4 c0 = make_float4(0.f, 0.f, 0.f, 0.f), c1 = c0;
+#pragma unroll
+  for (int k = 0; k < 8; k += 2) {
+    const int e0 = lane + 32 * k, e1 = e0 + 32;
+    if (e0 < n4) {
+      const float4 w = w4[e0], x = x4[e0];
+      c0.x = fmaf(w.x, x.x, c0.x);
+      c0.y = fmaf(w.y, x.y, c0.y);
+      c0.z = fmaf(w.z, x.z, c0.z);
+      c0.w = fmaf(w.w, x.w, c0.w);
+    }
+    if (e1 < n4) {
+      const float4 w = w4[e1], x = x4[e1];
+      c1.x = fmaf(w.x, x.x, c1.x);
+      c1.y = fmaf(w.y, x.y, c1.y);
+      c1.z = fmaf(w.z, x.z, c1.z);
+      c1.w = fmaf(w.w, x.w, c1.w);
+    }
+  }
+  return ((c0.x + c0.y) + (c0.z + c0.w)) + ((c1.x + c1.y) + (c1.z + c1.w));
+}
+
 // Consumer: one GEMV phase over the CTA's stage plan. The input vector xs is
 // in shared memory; with S > 1 the matrix is viewed as [M*S x Kc] "virtual
 // rows" (row r, K-chunk s) and virtual row v reads xs + (v % S) * Kc.
 // epi.store(v, value) receives each finished (virtual) row. Returns false on
 // abort, identically in every consumer thread (a barrier vote).
-template <class Epi>
-__device__ inline bool consume_phase(const Ring& r, uint32_t& g, const StagePlan& p,
+//
+// Work of one stage: its rows, each cut into P parts (P = 1, 2, 4 or 8, so
+// that short stages still give every warp a part); a part ("unit") is at most
+// 1024 floats: a row fits a stage (8192 floats), and P is chosen so that
+// rows x P >= 8 whenever a row is longer than 1024 floats. Warp w takes units
+// w, w+8, ...; each unit is one fully unrolled float4 stream and one shuffle
+// tree; a row adds its parts in order.
+template <class Epi, class Feed>
+__device__ inline bool consume_phase(const Ring& r, uint32_t& g, Feed& feed, const StagePlan& p,
                                      const float* xs, int S, int Kc, float* pdot, Epi& epi,
                                      int* err, int* err_host, volatile int* s_abort) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -195,41 +244,50 @@ __device__ inline bool consume_phase(const Ring& r, uint32_t& g, const StagePlan
     const bool ok = consumer_wait_full(&r.full[slot], par, err, err_host, s_abort);
     const StageDesc s = stage_desc(p, j);
     const int ncols = s.c1 - s.c0;
-    const int npr = (ncols + kPiece - 1) / kPiece;
-    const int npieces = s.nrows * npr;
+    int lp = 0;  // log2 of parts per row
+    while (lp < 3 && (s.nrows << lp) < kConsumerWarps && (ncols >> (lp + 1)) >= 128) ++lp;
+    const int units = s.nrows << lp;
+    const int U = (((ncols + (1 << lp) - 1) >> lp) + 3) & ~3;  // floats per part
     float* pd = pdot + (g & 1u) * kMaxPieces;
     if (ok) {
       const float* st = reinterpret_cast<const float*>(r.buf + (size_t)slot * kStageBytes);
-      for (int q = warp; q < npieces; q += kConsumerWarps) {
-        const int ri = q / npr, pj = q - ri * npr;
-        const int a = pj * kPiece;
-        const int b = (a + kPiece < ncols) ? a + kPiece : ncols;
+      auto unit = [&](int u) -> float {
+        const int ri = u >> lp, pj = u & ((1 << lp) - 1);
+        const int a = pj * U;
+        const int b = (a + U < ncols) ? a + U : ncols;
         const int v = s.row + ri;
         const float* xr = xs + (S > 1 ? (v % S) * Kc : 0) + s.c0 + a;
-        const float4* w4 = reinterpret_cast<const float4*>(st + (size_t)ri * ncols + a);
-        const float4* x4 = reinterpret_cast<const float4*>(xr);
-        const int n4 = (b - a) >> 2;
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int e = lane; e < n4; e += 32) {
-          const float4 w = w4[e], xv = x4[e];
-          acc.x = fmaf(w.x, xv.x, acc.x);
-          acc.y = fmaf(w.y, xv.y, acc.y);
-          acc.z = fmaf(w.z, xv.z, acc.z);
-          acc.w = fmaf(w.w, xv.w, acc.w);
+        return unit_partial(reinterpret_cast<const float4*>(st + (size_t)ri * ncols + a),
+                            reinterpret_cast<const float4*>(xr), (b - a) >> 2, lane);
+      };
+      // a warp takes units w and w+8 together: both loads in flight, both trees interleaved
+      for (int u = warp; u < units; u += 2 * kConsumerWarps) {
+        const bool two = u + kConsumerWarps < units;
+        float s0 = unit(u);
+        float s1 = two ? unit(u + kConsumerWarps) : 0.f;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          s0 += __shfl_xor_sync(0xffffffffu, s0, o);
+          s1 += __shfl_xor_sync(0xffffffffu, s1, o);
         }
-        const float sum = warp_sum((acc.x + acc.y) + (acc.z + acc.w));
-        if (lane == 0) pd[q] = sum;
+        if (lane == 0) {
+          pd[u] = s0;
+          if (two) pd[u + kConsumerWarps] = s1;
+        }
       }
     }
     // uniform decision: abort if any consumer thread gave up waiting
     if (named_bar_or(kBarConsumers, kConsumerThreads, !ok)) {
-      if (tid == 0) *s_abort = 1;
+      if (tid == 0) {
+        *s_abort = 1;
+        feed.drain(r, g);
+      }
       return false;
     }
-    if (tid == 0) mbar_arrive(&r.empty[slot]);  // stage free for the producer
+    if (tid == 0) feed.issue(r);  // the slot is free: queue the stage nst ahead
     for (int ri = tid; ri < s.nrows; ri += kConsumerThreads) {
       float v = 0.f;
-      for (int q = 0; q < npr; ++q) v += pd[ri * npr + q];
+      for (int q = 0; q < (1 << lp); ++q) v += pd[(ri << lp) + q];
       if (p.spr > 1) {  // a segment of one row: thread 0 carries the row sum
         const int k = j % p.spr;
         carry = (k == 0) ? v : carry + v;

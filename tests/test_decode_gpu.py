@@ -48,9 +48,9 @@ def test_tiny_model_64_steps(tvl):
     dict(n_kv_heads=2),                        # grouped query heads (2 query heads per kv head)
     dict(n_kv_heads=1, n_heads=8),             # one kv head, head_dim 8
     dict(n_layers=0),                          # embedding -> final norm -> classifier
-    dict(n_layers=1, hidden_dim=36, dim=32, n_heads=1, vocab_size=7),  # tiny vocab, one head
-    dict(dim=96, n_heads=2, hidden_dim=8200, vocab_size=333),          # W2 rows span two stages
-    dict(dim=128, n_heads=1, hidden_dim=256),  # head_dim 128
+    dict(n_layers=1, hidden_dim=36, dim=32, n_heads=1, n_kv_heads=1, vocab_size=7),  # one head
+    dict(dim=96, n_heads=2, n_kv_heads=2, hidden_dim=8200, vocab_size=333),  # W2 rows: 2 stages
+    dict(dim=128, n_heads=1, n_kv_heads=1, hidden_dim=256),  # head_dim 128
 ], ids=["base", "gqa2", "mqa", "L0", "v7", "wide_ffn", "hd128"])
 def test_small_shapes_match_oracle(tvl, kw):
     cfg = small_config(**kw)
