@@ -36,7 +36,7 @@ struct tvl_model {
 namespace {
 
 struct SmemPlan {
-  int ring, bars, xs, vec, pdot, att, misc, total, nst;
+  int ring, bars, xs, vec, seg, att, misc, total, nst;
 };
 
 SmemPlan plan_smem(int d, int F, int hd, int H, int nch_cap, int max_bytes) {
@@ -44,11 +44,11 @@ SmemPlan plan_smem(int d, int F, int hd, int H, int nch_cap, int max_bytes) {
   const int att_floats =
       std::max(3 * hd + kAttMaxChunk + 4 * kConsumerThreads, 2 * H * nch_cap) + 16;
   const int xs = (int)a128(4LL * d), vec = (int)a128(4LL * std::max(d, F));
-  const int pdot = 2 * kMaxPieces * 4, att = (int)a128(4LL * att_floats), misc = 256;
-  const int bars = 8 * 8;
-  const int other = bars + xs + vec + pdot + att + misc + 1024;  // + static shared memory
+  const int seg = kMaxSegParts * 4, att = (int)a128(4LL * att_floats), misc = 256;
+  const int bars = kRingBarBytes;
+  const int other = bars + xs + vec + seg + att + misc;
   int nst = (max_bytes - other) / kStageBytes;
-  if (nst > 8) nst = 8;
+  if (nst > kMaxStages) nst = kMaxStages;
   p.nst = nst;
   int off = 0;
   p.ring = off;
@@ -59,8 +59,8 @@ SmemPlan plan_smem(int d, int F, int hd, int H, int nch_cap, int max_bytes) {
   off += xs;
   p.vec = off;
   off += vec;
-  p.pdot = off;
-  off += pdot;
+  p.seg = off;
+  off += seg;
   p.att = off;
   off += att;
   p.misc = off;
@@ -188,6 +188,17 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   const int G = sms;
   const int nch_cap = nch_cap_for(S, H, G);
   const SmemPlan sp = plan_smem(d, F, hd, H, nch_cap, max_optin);
+  {  // segment partials of rows longer than a stage must fit the scratch
+    const long long Ms[5] = {d + 2LL * kvd, d, 2LL * F, d, V};
+    const int Ks[5] = {d, d, d, F, d};
+    for (int i = 0; i < 5; ++i) {
+      const StagePlan pl = plan_stages(Ms[i], Ks[i], G, 0);
+      if (pl.spr > 1 && (long long)((Ms[i] + G - 1) / G) * pl.spr > kMaxSegParts) {
+        set_error("tvl_load: too many long rows per SM for the segment scratch");
+        return fail(TVL_E_UNSUPPORTED);
+      }
+    }
+  }
   if (sp.nst < 2) {
     set_error("tvl_load: not enough shared memory for two weight stages");
     return fail(TVL_E_UNSUPPORTED);
@@ -329,7 +340,7 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   a.att_scale = (float)(1.0 / std::sqrt((double)hd));
   a.nst = sp.nst;
   a.sm_ring = sp.ring; a.sm_bars = sp.bars; a.sm_xs = sp.xs; a.sm_vec = sp.vec;
-  a.sm_pdot = sp.pdot; a.sm_att = sp.att; a.sm_misc = sp.misc;
+  a.sm_seg = sp.seg; a.sm_att = sp.att; a.sm_misc = sp.misc;
   a.wait_limit_ns = kWaitLimitNs;
   m->streamed_bytes =
       4LL * ((int64_t)L * ((int64_t)(d + 2 * kvd) * d + (int64_t)d * d + 3LL * F * d + 2LL * d) +

@@ -66,7 +66,7 @@ struct DecodeArgs {
   int start_token, start_pos, n_steps, final_token;
   unsigned epoch0;  // tag of the first exchange of this launch
   int nst;
-  int sm_ring, sm_bars, sm_xs, sm_vec, sm_pdot, sm_att, sm_misc;  // byte offsets
+  int sm_ring, sm_bars, sm_xs, sm_vec, sm_seg, sm_att, sm_misc;  // byte offsets
   unsigned long long wait_limit_ns;
 };
 
@@ -604,19 +604,18 @@ struct DecodeSched {
   }
 };
 
-using DecodeFeeder = Feeder<DecodeSched>;
-
-__device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, DecodeFeeder& feed,
-                                    uint32_t& g, unsigned char* smem, volatile int* s_abort) {
+__device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned char* smem,
+                                    volatile int* s_abort) {
   float* xs = reinterpret_cast<float*>(smem + a.sm_xs);
   float* vec = reinterpret_cast<float*>(smem + a.sm_vec);
-  float* pdot = reinterpret_cast<float*>(smem + a.sm_pdot);
+  float* seg = reinterpret_cast<float*>(smem + a.sm_seg);
   float* asm_ = reinterpret_cast<float*>(smem + a.sm_att);
   float* red = reinterpret_cast<float*>(smem + a.sm_misc) + 8;
   int* redi = reinterpret_cast<int*>(smem + a.sm_misc) + 24;
   const int tid = threadIdx.x, c = blockIdx.x;
   const Poll pc{a.err, a.err_host, s_abort, a.wait_limit_ns};
   const unsigned per_step = (unsigned)(kPhasesPerLayer * a.L + 1);
+  uint32_t g = 0;
   int token = a.start_token;
   // x += (published vector), identically in every CTA
   auto add_published = [&](const unsigned long long* src, unsigned tag) {
@@ -647,19 +646,19 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, DecodeFe
       if (l > 0 && !add_published(a.x_f, el - 1)) return false;
       rmsnorm_to(vec, xs, reinterpret_cast<const float*>(lw + a.o_gatt), a.d, a.eps, red);
       EpiTag e_qkv{a.x_qkv, el};
-      if (!consume_phase(r, g, feed, plan_stages(a.d + 2 * a.kvd, a.d, a.G, c), vec, 1, a.d, pdot,
+      if (!consume_phase<false>(r, g, plan_stages(a.d + 2 * a.kvd, a.d, a.G, c), vec, 1, a.d, seg,
                          e_qkv, a.err, a.err_host, s_abort))
         return false;
       if (!attention_phase(a, l, pos, el, el + 1, asm_, red, pc)) return false;
       if (!merge_attention(a, pos, el + 1, vec, asm_, pc)) return false;
       EpiTag e_o{a.x_o, el + 2};
-      if (!consume_phase(r, g, feed, plan_stages(a.d, a.d, a.G, c), vec, 1, a.d, pdot, e_o, a.err,
+      if (!consume_phase<false>(r, g, plan_stages(a.d, a.d, a.G, c), vec, 1, a.d, seg, e_o, a.err,
                          a.err_host, s_abort))
         return false;
       if (!add_published(a.x_o, el + 2)) return false;
       rmsnorm_to(vec, xs, reinterpret_cast<const float*>(lw + a.o_gffn), a.d, a.eps, red);
       EpiTag e_13{a.x_h13, el + 3};
-      if (!consume_phase(r, g, feed, plan_stages(2 * a.F, a.d, a.G, c), vec, 1, a.d, pdot, e_13, a.err,
+      if (!consume_phase<false>(r, g, plan_stages(2 * a.F, a.d, a.G, c), vec, 1, a.d, seg, e_13, a.err,
                          a.err_host, s_abort))
         return false;
       {  // h = silu(a) * b (paper §2.1, SwiGLU); a = h13[k], b = h13[F + k]
@@ -671,14 +670,14 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, DecodeFe
         if (!vote_ok(ok, s_abort)) return false;
       }
       EpiTag e_2{a.x_f, el + 4};
-      if (!consume_phase(r, g, feed, plan_stages(a.d, a.F, a.G, c), vec, 1, a.F, pdot, e_2, a.err,
+      if (!consume_phase<false>(r, g, plan_stages(a.d, a.F, a.G, c), vec, 1, a.F, seg, e_2, a.err,
                          a.err_host, s_abort))
         return false;
     }
     if (a.L > 0 && !add_published(a.x_f, es + per_step - 2)) return false;
     rmsnorm_to(vec, xs, a.g_final, a.d, a.eps, red);
     EpiArgmax ea{a.logits, -INFINITY, 0x7fffffff};
-    if (!consume_phase(r, g, feed, plan_stages(a.V, a.d, a.G, c), vec, 1, a.d, pdot, ea, a.err,
+    if (!consume_phase<false>(r, g, plan_stages(a.V, a.d, a.G, c), vec, 1, a.d, seg, ea, a.err,
                        a.err_host, s_abort))
       return false;
     float bv = ea.bv;
@@ -708,20 +707,29 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
   Ring r;
   r.buf = smem + a.sm_ring;
   r.full = reinterpret_cast<uint64_t*>(smem + a.sm_bars);
+  r.empty = r.full + a.nst;
+  r.seq = reinterpret_cast<volatile int*>(r.empty + a.nst);
   r.nst = a.nst;
   volatile int* s_abort = reinterpret_cast<volatile int*>(smem + a.sm_misc);
-  __shared__ DecodeFeeder feed;
   if (threadIdx.x == 0) {
-    feed = DecodeFeeder();
-    feed.sched.a = &a;
-    for (int i = 0; i < a.nst; ++i) mbar_init(&r.full[i], 1);
+    for (int i = 0; i < a.nst; ++i) {
+      mbar_init(&r.full[i], 1);
+      mbar_init(&r.empty[i], 1);
+      r.seq[i] = 0;
+    }
     *s_abort = 0;
     fence_mbar_init();
-    feed.start(r);
   }
   __syncthreads();
-  uint32_t g = 0;
-  if (!decode_steps(a, r, feed, g, smem, s_abort) && threadIdx.x == 0) feed.drain(r, g);
+  if (threadIdx.x >= kConsumerThreads) {
+    if (threadIdx.x == kConsumerThreads) {
+      DecodeSched sched;
+      sched.a = &a;
+      run_producer(r, sched, a.err, a.err_host, s_abort);
+    }
+    return;
+  }
+  decode_steps(a, r, smem, s_abort);
 }
 
 // Failure-detection self-test: one CTA polls a tagged word that nothing
@@ -731,7 +739,7 @@ __global__ void wait_selftest_kernel(unsigned long long* word, int* err,
   __shared__ int s_abort;
   if (threadIdx.x == 0) s_abort = 0;
   __syncthreads();
-  if (threadIdx.x >= kConsumerThreads) return;
+  if (threadIdx.x >= kConsumerThreads) return;  // the consumer warps take part
   const Poll pc{err, nullptr, &s_abort, limit_ns};
   const bool ok = poll_pairs(word, 1, 1u, pc, [](int, float, float) {});
   vote_ok(ok, &s_abort);

@@ -1,7 +1,7 @@
 // gemv.cu — standalone y = W x (paper §6.1) on the weight-streaming engine.
 //
 // One CTA per SM streams its contiguous share of W through the shared-memory
-// stage ring (8 warps; thread 0 keeps the ring full). Matrices with few rows are split along K into S chunks so that
+// stage ring (a producer warp and seven consumer warps). Matrices with few rows are split along K into S chunks so that
 // every SM gets work: virtual row v = (row v / S, chunk v % S); each virtual
 // row's partial lands in a scratch buffer, and each row is summed over its
 // S chunks in chunk order — by the CTA that owns the whole row, or for a row
@@ -29,7 +29,7 @@ struct GemvArgs {
   float* part;   // [M * S] when S > 1
   int* cnt;      // [M], zero between calls
   int nst;
-  int sm_ring, sm_bars, sm_x, sm_pdot, sm_misc;
+  int sm_ring, sm_bars, sm_x, sm_seg, sm_misc;
 };
 
 struct EpiPart {
@@ -56,35 +56,42 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   Ring r;
   r.buf = smem + a.sm_ring;
   r.full = reinterpret_cast<uint64_t*>(smem + a.sm_bars);
+  r.empty = r.full + a.nst;
+  r.seq = reinterpret_cast<volatile int*>(r.empty + a.nst);
   r.nst = a.nst;
   volatile int* s_abort = reinterpret_cast<volatile int*>(smem + a.sm_misc);
   const StagePlan p = plan_stages(a.nv, a.Kc, gridDim.x, blockIdx.x);
-  __shared__ Feeder<GemvSched> feed;
   if (threadIdx.x == 0) {
-    feed = Feeder<GemvSched>();
-    feed.sched.W = a.W;
-    feed.sched.p = p;
-    feed.sched.given = false;
-    for (int i = 0; i < a.nst; ++i) mbar_init(&r.full[i], 1);
+    for (int i = 0; i < a.nst; ++i) {
+      mbar_init(&r.full[i], 1);
+      mbar_init(&r.empty[i], 1);
+      r.seq[i] = 0;
+    }
     *s_abort = 0;
     fence_mbar_init();
-    feed.start(r);
   }
   __syncthreads();
   uint32_t g = 0;
+  if (threadIdx.x >= kConsumerThreads) {
+    if (threadIdx.x == kConsumerThreads) {
+      GemvSched sched{a.W, p, false};
+      run_producer(r, sched, nullptr, nullptr, s_abort);
+    }
+    return;
+  }
   float* xs = reinterpret_cast<float*>(smem + a.sm_x);
-  float* pdot = reinterpret_cast<float*>(smem + a.sm_pdot);
+  float* seg = reinterpret_cast<float*>(smem + a.sm_seg);
   const float4* x4 = reinterpret_cast<const float4*>(a.x);
   for (int j = threadIdx.x; j < (a.K >> 2); j += kConsumerThreads)
     reinterpret_cast<float4*>(xs)[j] = __ldg(x4 + j);
   named_bar_sync(kBarConsumers, kConsumerThreads);
   if (a.S == 1) {
     EpiStore e{a.y};
-    consume_phase(r, g, feed, p, xs, 1, a.Kc, pdot, e, nullptr, nullptr, s_abort);
+    consume_phase(r, g, p, xs, 1, a.Kc, seg, e, nullptr, nullptr, s_abort);
     return;
   }
   EpiPart e{a.part};
-  if (!consume_phase(r, g, feed, p, xs, a.S, a.Kc, pdot, e, nullptr, nullptr, s_abort)) return;
+  if (!consume_phase(r, g, p, xs, a.S, a.Kc, seg, e, nullptr, nullptr, s_abort)) return;
   if (p.r1 <= p.r0) return;
   named_bar_sync(kBarConsumers, kConsumerThreads);
   const int S = a.S;
@@ -168,7 +175,15 @@ extern "C" tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t
     info = di;
   }
   const bool aligned = ((uintptr_t)W % 16 == 0) && ((uintptr_t)x % 16 == 0) && d_in % 4 == 0;
-  if (!aligned || d_in > 16384) {
+  bool fits = aligned && d_in <= 16384;
+  if (fits) {  // segment partials of rows longer than a stage must fit the scratch
+    const int S = split_for(d_out, d_in, info.sms);
+    const long long nv = (long long)d_out * S;
+    const StagePlan pl = plan_stages(nv, d_in / S, (int)(nv < info.sms ? nv : info.sms), 0);
+    const long long G = nv < info.sms ? nv : info.sms;
+    fits = pl.spr == 1 || ((nv + G - 1) / G) * pl.spr <= kMaxSegParts;
+  }
+  if (!fits) {
     const int threads = 256, rows_per_block = threads / 32;
     gemv_rowwise_kernel<<<(d_out + rows_per_block - 1) / rows_per_block, threads, 0, s>>>(
         W, x, y, d_out, d_in);
@@ -186,10 +201,10 @@ extern "C" tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t
   a.nv = (long long)d_out * a.S;
   const int G = (int)(a.nv < info.sms ? a.nv : info.sms);
   // shared memory: ring | barriers | x | piece sums | misc
-  const int xbytes = (int)a128(4LL * d_in), pdot = 2 * kMaxPieces * 4, bars = 128, misc = 128;
-  // (minus 1 KB for the kernel's static shared memory)
-  int nst = (info.max_optin - 1024 - xbytes - pdot - bars - misc) / kStageBytes;
-  if (nst > 6) nst = 6;
+  const int xbytes = (int)a128(4LL * d_in), segb = kMaxSegParts * 4, bars = kRingBarBytes;
+  const int misc = 128;
+  int nst = (info.max_optin - xbytes - segb - bars - misc) / kStageBytes;
+  if (nst > kMaxStages) nst = kMaxStages;
   if (nst < 2) {
     set_error("tvl_gemv: not enough shared memory");
     return TVL_E_UNSUPPORTED;
@@ -198,8 +213,8 @@ extern "C" tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t
   a.sm_ring = 0;
   a.sm_bars = nst * kStageBytes;
   a.sm_x = a.sm_bars + bars;
-  a.sm_pdot = a.sm_x + xbytes;
-  a.sm_misc = a.sm_pdot + pdot;
+  a.sm_seg = a.sm_x + xbytes;
+  a.sm_misc = a.sm_seg + segb;
   const int smem = a.sm_misc + misc;
   {
     std::lock_guard<std::mutex> lk(g_ws_mu);

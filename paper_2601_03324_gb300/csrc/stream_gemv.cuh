@@ -2,35 +2,42 @@
 // kernel and the standalone GEMV (paper §3.1: y = W x reads every weight once,
 // so the work is bound by memory; §6.1: one dot product per output row).
 //
-// Per CTA: a ring of shared-memory stages is filled with bulk asynchronous
-// copies (the TMA engine) of a contiguous range of weight rows, each stage
-// completing on an mbarrier; eight warps multiply each landed stage by the
-// input vector held in shared memory. Thread 0 keeps the ring full: it issues
-// the copy of stage g + nst as soon as stage g is consumed, walking a static
-// schedule of phases that does not depend on activations, so the copies run
-// ahead of whatever the warps are waiting for. This is the GPU form of the paper's two memory ideas: the
+// Per CTA: a producer warp fills a ring of shared-memory stages with bulk
+// asynchronous copies (the TMA engine) of a contiguous range of weight rows,
+// each stage completing on an mbarrier; seven consumer warps multiply each
+// landed stage by the input vector held in shared memory and hand the stage
+// back through a second mbarrier. The producer walks a static schedule of
+// phases that does not depend on activations, so the copies run ahead of
+// whatever the consumers are waiting for. (Eight warps in all: two per SM
+// sub-partition, which leaves each thread up to 255 registers; a ninth warp
+// would put three warps on one sub-partition and cap them at 168.) The
+// producer is a warp of its own because issuing a bulk copy can stall when
+// the copy engine's queue is full, and that stall must not hold up the math. This is the GPU form of the paper's two memory ideas: the
 // weights flow as one aligned stream (§3.2, §4.1) and several independent
 // loads are always in flight (§11.1's four accumulators become several
 // 32 KB stages in flight per SM).
 //
 // Work split: CTA c owns rows [M*c/G, M*(c+1)/G) of an [M x K] matrix, which
-// is one contiguous byte range. A stage holds whole rows (when a row fits in
-// a stage) or one segment of a row. Inside a stage, each row is one unit of
-// work for a warp, or 2/4/8 parts when the stage has fewer rows than warps;
-// each unit sum is a fixed shuffle tree and each row sums its parts in order,
-// so the result is bit-reproducible.
+// is one contiguous byte range. A stage (16 KB) holds whole rows, or one
+// segment of a row longer than a stage. Stage g of the CTA belongs to consumer
+// warp g mod 7, which waits for it, computes its rows (two at a time, one
+// float4 stream per lane and one shuffle tree per row), stores the results and
+// hands the stage back: the warps work on different stages at once and meet
+// only at the end of a phase. Segment partial sums of long rows are added in
+// segment order at that point, so every result is bit-reproducible.
 #pragma once
 #include "ptx.cuh"
 
 namespace tvl {
 
-constexpr int kConsumerWarps = 8;
+constexpr int kConsumerWarps = 7;
 constexpr int kConsumerThreads = kConsumerWarps * 32;
-constexpr int kThreads = kConsumerThreads;  // 2 warps per SM sub-partition: up to 255 registers
-constexpr int kStageBytes = 32768;
+constexpr int kThreads = kConsumerThreads + 32;  // + the producer warp
+constexpr int kStageBytes = 16384;
 constexpr int kStageFloats = kStageBytes / 4;
 constexpr int kMaxRowsPerStage = 256;
-constexpr int kMaxPieces = 256;       // per stage; see plan_stages
+constexpr int kMaxSegParts = 2048;    // segment partials of one phase (rows x segments)
+constexpr int kMaxStages = 12;        // ring slots
 constexpr uint32_t kBarConsumers = 1; // named barrier of the consumer warps
 constexpr unsigned long long kWaitLimitNs = 1000000000ull;  // 1 s per wait
 
@@ -51,8 +58,7 @@ struct StageDesc {
 };
 
 // Requires K % 4 == 0 (16-byte rows) and kStageFloats % 32 == 0. A stage has
-// at most kMaxRowsPerStage rows; units per stage (rows x parts) stay below
-// max(kMaxRowsPerStage, 2 * kConsumerWarps) <= kMaxPieces.
+// at most kMaxRowsPerStage rows, or one segment of at most kStageFloats.
 __host__ __device__ inline StagePlan plan_stages(long long M, int K, int G, int c) {
   StagePlan p;
   p.r0 = (int)(M * c / G);
@@ -60,8 +66,14 @@ __host__ __device__ inline StagePlan plan_stages(long long M, int K, int G, int 
   p.K = K;
   const int nrows = p.r1 - p.r0;
   if (K <= kStageFloats) {
-    p.rps = kStageFloats / K;
-    if (p.rps > kMaxRowsPerStage) p.rps = kMaxRowsPerStage;
+    // rows per stage: as many as fit, but few enough that the CTA's rows of
+    // this phase spread over all consumer warps (a phase's latency is that of
+    // its busiest warp)
+    int cap = kStageFloats / K;
+    if (cap > kMaxRowsPerStage) cap = kMaxRowsPerStage;
+    int spread = (nrows + kConsumerWarps - 1) / kConsumerWarps;
+    if (spread < 1) spread = 1;
+    p.rps = spread < cap ? spread : cap;
     p.spr = 1;
     p.seg = K;
     p.nstages = (nrows + p.rps - 1) / p.rps;
@@ -93,9 +105,14 @@ __host__ __device__ inline StageDesc stage_desc(const StagePlan& p, int j) {
 
 struct Ring {
   unsigned char* buf;
-  uint64_t* full;  // [nst]
+  uint64_t* full;     // [nst] stage landed
+  uint64_t* empty;    // [nst] stage consumed
+  volatile int* seq;  // [nst] 1 + number of the stage last queued into the slot
   int nst;
 };
+
+// Shared-memory bytes of a ring's barriers and sequence numbers.
+constexpr int kRingBarBytes = 3 * kMaxStages * 8;
 
 __device__ __forceinline__ void raise_error(int* err, int* err_host, int code) {
   if (err) atomicCAS(err, 0, code);
@@ -120,57 +137,54 @@ __device__ inline bool wait_bounded(uint64_t* bar, uint32_t par, const int* err,
   }
 }
 
-// Queues the stages of a static schedule of GEMV phases into the ring, in
-// order. Sched::next(W, plan) yields the next phase's matrix and this CTA's
-// stage plan, false at the end. Used by thread 0 only; the object lives in
-// shared memory so that its state takes no registers in the stage loop.
+// Producer: queue the stages of a static schedule of GEMV phases into the
+// ring, in order. Sched::next(W, plan) yields the next phase's matrix and this
+// CTA's stage plan, false at the end. Before reusing a slot it waits for the
+// consumers to release it; before returning it waits for every copy it queued
+// (a CTA must not exit with copies into its shared memory in flight).
 template <class Sched>
-struct Feeder {
-  Sched sched;
+__device__ inline void run_producer(const Ring& r, Sched& sched, int* err, int* err_host,
+                                    volatile int* s_abort) {
+  const uint64_t pol = l2_evict_first();
+  uint32_t g = 0;
   const float* W = nullptr;
-  StagePlan p{};
-  int j = 0;            // next stage of the current phase
-  uint32_t issued = 0;  // stages queued so far
-  bool done = false;
-  uint64_t pol = 0;
-
-  __device__ void start(const Ring& r) {
-    pol = l2_evict_first();
-    p.nstages = 0;
-    for (int k = 0; k < r.nst; ++k) issue(r);
-  }
-  // Queue the next stage into slot issued % nst (its previous stage has been
-  // consumed: the caller has passed the barrier that ends it).
-  __device__ void issue(const Ring& r) {
-    if (done) return;
-    while (j >= p.nstages) {
-      if (!sched.next(W, p)) {
-        done = true;
-        return;
+  StagePlan p;
+  bool ok = true;
+  while (ok && sched.next(W, p)) {
+    for (int j = 0; j < p.nstages; ++j, ++g) {
+      const int slot = (int)(g % (uint32_t)r.nst);
+      if (g >= (uint32_t)r.nst) {
+        bool to = false;
+        const uint32_t par = ((g / (uint32_t)r.nst) - 1u) & 1u;
+        if (!wait_bounded(&r.empty[slot], par, err, s_abort, true, &to)) {
+          if (to) raise_error(err, err_host, kErrTimeout);
+          *s_abort = 1;
+          ok = false;
+          break;
+        }
       }
-      j = 0;
+      const StageDesc s = stage_desc(p, j);
+      const uint32_t bytes = (uint32_t)(s.nrows * (s.c1 - s.c0)) * 4u;
+      mbar_arrive_expect_tx(&r.full[slot], bytes);
+      bulk_g2s(r.buf + (size_t)slot * kStageBytes, W + (size_t)s.row * p.K + s.c0, bytes,
+               &r.full[slot], pol);
+      // The slot's barrier is now in this stage's phase: say so. Consumers
+      // take stages out of order, and a parity wait is only meaningful once
+      // the barrier has reached the awaited phase.
+      __threadfence_block();
+      r.seq[slot] = (int)(g + 1u);
     }
-    const StageDesc s = stage_desc(p, j);
-    const uint32_t bytes = (uint32_t)(s.nrows * (s.c1 - s.c0)) * 4u;
-    const int slot = (int)(issued % (uint32_t)r.nst);
-    mbar_arrive_expect_tx(&r.full[slot], bytes);
-    bulk_g2s(r.buf + (size_t)slot * kStageBytes, W + (size_t)s.row * p.K + s.c0, bytes,
-             &r.full[slot], pol);
-    ++j;
-    ++issued;
   }
-  // Before the CTA leaves early: wait for the copies still in flight.
-  __device__ void drain(const Ring& r, uint32_t consumed) {
-    for (uint32_t k = consumed; k < issued; ++k)
-      wait_bounded(&r.full[k % (uint32_t)r.nst], (k / (uint32_t)r.nst) & 1u, nullptr, nullptr,
-                   false, nullptr);
-  }
-};
+  const uint32_t from = g > (uint32_t)r.nst ? g - (uint32_t)r.nst : 0u;
+  for (uint32_t k = from; k < g; ++k)
+    wait_bounded(&r.full[k % (uint32_t)r.nst], (k / (uint32_t)r.nst) & 1u, nullptr, nullptr,
+                 false, nullptr);
+}
 
-// All threads poll; thread 0 alone applies the limit and raises the abort
-// flag, which the others observe. Returns true if the stage landed. The flag
-// is only a hint to stop waiting: the decision to leave is taken by a vote at
-// the next barrier.
+// All consumer threads poll; thread 0 alone applies the limit and raises the
+// abort flag, which the others observe (the producer may raise it too).
+// Returns true if the stage landed. The flag is only a hint to stop waiting:
+// the decision to leave is taken by a vote at the next barrier.
 __device__ inline bool consumer_wait_full(uint64_t* bar, uint32_t par, int* err, int* err_host,
                                           volatile int* s_abort) {
   if (mbar_try_wait(bar, par)) return true;
@@ -193,109 +207,198 @@ __device__ inline bool consumer_wait_full(uint64_t* bar, uint32_t par, int* err,
   }
 }
 
-// Lane part of one unit's dot product: n4 <= 256 float4 of weights and
-// input; lane takes float4 lane + 32k (k < 8), in a fully unrolled loop whose
-// loads the compiler hoists as far as registers allow.
-__device__ __forceinline__ float unit_partial(const float4* w4, const float4* x4, int n4,
-                                              int lane) {
+// Lane part of one row's dot product: n4 float4 of weights (shared memory)
+// and input; lane takes float4 lane, lane + 32, ...
+__device__ __forceinline__ float row_partial(const float4* w4, const float4* x4, int n4,
+                                             int lane) {
+  float4 c0 = make_float4(0.f, 0.f, 0.f, 0.f), c1 = c0;
+  int e = lane;
+#pragma unroll 2
+  for (; e + 32 < n4; e += 64) {
+    const float4 w0 = w4[e], x0 = x4[e], w1 = w4[e + 32], x1 = x4[e + 32];
+    c0.x = fmaf(w0.x, x0.x, c0.x);
+    c0.y = fmaf(w0.y, x0.y, c0.y);
+    c0.z = fmaf(w0.z, x0.z, c0.z);
+    c0.w = fmaf(w0.w, x0.w, c0.w);
+    c1.x = fmaf(w1.x, x1.x, c1.x);
+    c1.y = fmaf(w1.y, x1.y, c1.y);
+    c1.z = fmaf(w1.z, x1.z, c1.z);
+    c1.w = fmaf(w1.w, x1.w, c1.w);
+  }
+  if (e < n4) {
+    const float4 w0 = w4[e], x0 = x4[e];
+    c0.x = fmaf(w0.x, x0.x, c0.x);
+    c0.y = fmaf(w0.y, x0.y, c0.y);
+    c0.z = fmaf(w0.z, x0.z, c0.z);
+    c0.w = fmaf(w0.w, x0.w, c0.w);
+  }
+  return ((c0.x + c0.y) + (c0.z + c0.w)) + ((c1.x + c1.y) + (c1.z + c1.w));
+}
+
+// Same for rows of at most 1024 floats with the lane's slice of x already in
+// registers: xr[k] holds x float4 lane + 32k.
+__device__ __forceinline__ float row_partial_xr(const float4* w4, const float4 (&xr)[8], int n4,
+                                                int lane) {
   float4 c0 = make_float4(0.f, 0.f, 0.f, 0.f), c1 = c0;
 #pragma unroll
   for (int k = 0; k < 8; k += 2) {
-    const int e0 = lane + 32 * k, e1 = e0 + 32;
-    if (e0 < n4) {
-      const float4 w = w4[e0], x = x4[e0];
-      c0.x = fmaf(w.x, x.x, c0.x);
-      c0.y = fmaf(w.y, x.y, c0.y);
-      c0.z = fmaf(w.z, x.z, c0.z);
-      c0.w = fmaf(w.w, x.w, c0.w);
+    if (lane + 32 * k < n4) {
+      const float4 w = w4[lane + 32 * k];
+      c0.x = fmaf(w.x, xr[k].x, c0.x);
+      c0.y = fmaf(w.y, xr[k].y, c0.y);
+      c0.z = fmaf(w.z, xr[k].z, c0.z);
+      c0.w = fmaf(w.w, xr[k].w, c0.w);
     }
-    if (e1 < n4) {
-      const float4 w = w4[e1], x = x4[e1];
-      c1.x = fmaf(w.x, x.x, c1.x);
-      c1.y = fmaf(w.y, x.y, c1.y);
-      c1.z = fmaf(w.z, x.z, c1.z);
-      c1.w = fmaf(w.w, x.w, c1.w);
+    if (lane + 32 * (k + 1) < n4) {
+      const float4 w = w4[lane + 32 * (k + 1)];
+      c1.x = fmaf(w.x, xr[k + 1].x, c1.x);
+      c1.y = fmaf(w.y, xr[k + 1].y, c1.y);
+      c1.z = fmaf(w.z, xr[k + 1].z, c1.z);
+      c1.w = fmaf(w.w, xr[k + 1].w, c1.w);
     }
   }
   return ((c0.x + c0.y) + (c0.z + c0.w)) + ((c1.x + c1.y) + (c1.z + c1.w));
 }
 
+// Warp-level bounded wait for stage gs in `slot` (all lanes poll, lane 0
+// applies the limit): first until the producer has queued that stage into the
+// slot, then until its bytes have landed. Returns the same answer in every
+// lane of the warp.
+__device__ inline bool warp_wait_full(const Ring& r, int slot, uint32_t gs, int* err,
+                                      int* err_host, volatile int* s_abort) {
+  uint64_t* bar = &r.full[slot];
+  const uint32_t par = (gs / (uint32_t)r.nst) & 1u;
+  bool ok = true;
+  if (r.seq[slot] != (int)(gs + 1u)) {
+    const bool leader = (threadIdx.x & 31) == 0;
+    const uint64_t t0 = leader ? globaltimer_ns() : 0;
+    for (uint32_t it = 1; r.seq[slot] != (int)(gs + 1u); ++it) {
+      if (*s_abort) {
+        ok = false;
+        break;
+      }
+      if (leader && (it & 15u) == 0) {
+        if ((err && ld_volatile_s32(err)) || globaltimer_ns() - t0 > kWaitLimitNs ||
+            it > (1u << 26)) {
+          if (!(err && ld_volatile_s32(err))) raise_error(err, err_host, kErrTimeout);
+          *s_abort = 1;
+          ok = false;
+          break;
+        }
+      }
+    }
+  }
+  __threadfence_block();
+  if (!__any_sync(0xffffffffu, !ok)) ok = true;
+  else return false;
+  if (!mbar_try_wait(bar, par)) {
+    const bool leader = (threadIdx.x & 31) == 0;
+    const uint64_t t0 = leader ? globaltimer_ns() : 0;
+    for (uint32_t it = 1;; ++it) {
+      if (mbar_try_wait(bar, par)) break;
+      if (*s_abort) {
+        ok = false;
+        break;
+      }
+      if (leader && (it & 15u) == 0) {
+        if ((err && ld_volatile_s32(err)) || globaltimer_ns() - t0 > kWaitLimitNs ||
+            it > (1u << 26)) {
+          if (!(err && ld_volatile_s32(err))) raise_error(err, err_host, kErrTimeout);
+          *s_abort = 1;
+          ok = false;
+          break;
+        }
+      }
+    }
+  }
+  return !__any_sync(0xffffffffu, !ok);
+}
+
 // Consumer: one GEMV phase over the CTA's stage plan. The input vector xs is
 // in shared memory; with S > 1 the matrix is viewed as [M*S x Kc] "virtual
 // rows" (row r, K-chunk s) and virtual row v reads xs + (v % S) * Kc.
-// epi.store(v, value) receives each finished (virtual) row. Returns false on
-// abort, identically in every consumer thread (a barrier vote).
-//
-// Work of one stage: its rows, each cut into P parts (P = 1, 2, 4 or 8, so
-// that short stages still give every warp a part); a part ("unit") is at most
-// 1024 floats: a row fits a stage (8192 floats), and P is chosen so that
-// rows x P >= 8 whenever a row is longer than 1024 floats. Warp w takes units
-// w, w+8, ...; each unit is one fully unrolled float4 stream and one shuffle
-// tree; a row adds its parts in order.
-template <class Epi, class Feed>
-__device__ inline bool consume_phase(const Ring& r, uint32_t& g, Feed& feed, const StagePlan& p,
-                                     const float* xs, int S, int Kc, float* pdot, Epi& epi,
+// epi.store(v, value) receives each finished (virtual) row, from lane 0 of
+// the warp that computed it, or (rows longer than a stage) from the thread
+// that adds the row's segment partials at the end of the phase. seg is
+// shared scratch for those partials. Ends with a barrier of the consumer
+// warps; returns false on abort, identically in every consumer thread.
+template <bool kXReg = true, class Epi>
+__device__ inline bool consume_phase(const Ring& r, uint32_t& g, const StagePlan& p,
+                                     const float* xs, int S, int Kc, float* seg, Epi& epi,
                                      int* err, int* err_host, volatile int* s_abort) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  float carry = 0.f;
-  for (int j = 0; j < p.nstages; ++j, ++g) {
-    const int slot = (int)(g % (uint32_t)r.nst);
-    const uint32_t par = (g / (uint32_t)r.nst) & 1u;
-    const bool ok = consumer_wait_full(&r.full[slot], par, err, err_host, s_abort);
-    const StageDesc s = stage_desc(p, j);
-    const int ncols = s.c1 - s.c0;
-    int lp = 0;  // log2 of parts per row
-    while (lp < 3 && (s.nrows << lp) < kConsumerWarps && (ncols >> (lp + 1)) >= 128) ++lp;
-    const int units = s.nrows << lp;
-    const int U = (((ncols + (1 << lp) - 1) >> lp) + 3) & ~3;  // floats per part
-    float* pd = pdot + (g & 1u) * kMaxPieces;
-    if (ok) {
-      const float* st = reinterpret_cast<const float*>(r.buf + (size_t)slot * kStageBytes);
-      auto unit = [&](int u) -> float {
-        const int ri = u >> lp, pj = u & ((1 << lp) - 1);
-        const int a = pj * U;
-        const int b = (a + U < ncols) ? a + U : ncols;
-        const int v = s.row + ri;
-        const float* xr = xs + (S > 1 ? (v % S) * Kc : 0) + s.c0 + a;
-        return unit_partial(reinterpret_cast<const float4*>(st + (size_t)ri * ncols + a),
-                            reinterpret_cast<const float4*>(xr), (b - a) >> 2, lane);
-      };
-      // a warp takes units w and w+8 together: both loads in flight, both trees interleaved
-      for (int u = warp; u < units; u += 2 * kConsumerWarps) {
-        const bool two = u + kConsumerWarps < units;
-        float s0 = unit(u);
-        float s1 = two ? unit(u + kConsumerWarps) : 0.f;
+  // Rows of at most 1024 floats (whole rows in a stage, one K-chunk): each lane
+  // keeps its x slice in registers for the whole phase.
+  const bool xreg = kXReg && (p.spr == 1) && (p.K <= 1024) && (S == 1);
+  float4 xr[8];
+  if (xreg) {
+    const float4* x4 = reinterpret_cast<const float4*>(xs);
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-          s0 += __shfl_xor_sync(0xffffffffu, s0, o);
-          s1 += __shfl_xor_sync(0xffffffffu, s1, o);
-        }
-        if (lane == 0) {
-          pd[u] = s0;
-          if (two) pd[u + kConsumerWarps] = s1;
-        }
-      }
+    for (int k = 0; k < 8; ++k) {
+      const int e = lane + 32 * k;
+      xr[k] = (e < (p.K >> 2)) ? x4[e] : make_float4(0.f, 0.f, 0.f, 0.f);
     }
-    // uniform decision: abort if any consumer thread gave up waiting
-    if (named_bar_or(kBarConsumers, kConsumerThreads, !ok)) {
-      if (tid == 0) {
-        *s_abort = 1;
-        feed.drain(r, g);
-      }
-      return false;
+  }
+  bool ok = true;
+  // this warp's stages of the phase: global stage numbers g + j with (g + j) % 7 == warp
+  int j = (int)((warp + kConsumerWarps - (int)(g % kConsumerWarps)) % kConsumerWarps);
+  for (; j < p.nstages && ok; j += kConsumerWarps) {
+    const uint32_t gs = g + (uint32_t)j;
+    const int slot = (int)(gs % (uint32_t)r.nst);
+    if (!warp_wait_full(r, slot, gs, err, err_host, s_abort)) {
+      ok = false;
+      break;
     }
-    if (tid == 0) feed.issue(r);  // the slot is free: queue the stage nst ahead
-    for (int ri = tid; ri < s.nrows; ri += kConsumerThreads) {
-      float v = 0.f;
-      for (int q = 0; q < (1 << lp); ++q) v += pd[(ri << lp) + q];
-      if (p.spr > 1) {  // a segment of one row: thread 0 carries the row sum
-        const int k = j % p.spr;
-        carry = (k == 0) ? v : carry + v;
-        if (k == p.spr - 1) epi.store(s.row, carry);
+    const StageDesc s = stage_desc(p, j);
+    const int ncols = s.c1 - s.c0, n4 = ncols >> 2;
+    const float* st = reinterpret_cast<const float*>(r.buf + (size_t)slot * kStageBytes);
+    for (int ri = 0; ri < s.nrows; ri += 2) {
+      const bool two = ri + 1 < s.nrows;
+      const int v0 = s.row + ri, v1 = v0 + 1;
+      const float4* w0 = reinterpret_cast<const float4*>(st + (size_t)ri * ncols);
+      const float4* w1 = w0 + n4;
+      float a0, a1 = 0.f;
+      if (xreg) {
+        a0 = row_partial_xr(w0, xr, n4, lane);
+        if (two) a1 = row_partial_xr(w1, xr, n4, lane);
       } else {
-        epi.store(s.row + ri, v);
+        const float* xb = xs + s.c0;
+        a0 = row_partial(w0, reinterpret_cast<const float4*>(xb + (S > 1 ? (v0 % S) * Kc : 0)),
+                         n4, lane);
+        if (two)
+          a1 = row_partial(w1, reinterpret_cast<const float4*>(xb + (S > 1 ? (v1 % S) * Kc : 0)),
+                           n4, lane);
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        a0 += __shfl_xor_sync(0xffffffffu, a0, o);
+        a1 += __shfl_xor_sync(0xffffffffu, a1, o);
+      }
+      if (lane == 0) {
+        if (p.spr > 1) {
+          seg[(v0 - p.r0) * p.spr + j % p.spr] = a0;
+        } else {
+          epi.store(v0, a0);
+          if (two) epi.store(v1, a1);
+        }
       }
     }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&r.empty[slot]);  // stage free for the producer
+  }
+  g += (uint32_t)p.nstages;
+  // every stage of the phase is consumed (or the CTA gives up together)
+  if (named_bar_or(kBarConsumers, kConsumerThreads, !ok)) {
+    if (tid == 0) *s_abort = 1;
+    return false;
+  }
+  if (p.spr > 1) {  // rows longer than a stage: add the segments in order
+    for (int ri = tid; ri < p.r1 - p.r0; ri += kConsumerThreads) {
+      float v = 0.f;
+      for (int k = 0; k < p.spr; ++k) v += seg[ri * p.spr + k];
+      epi.store(p.r0 + ri, v);
+    }
+    named_bar_sync(kBarConsumers, kConsumerThreads);
   }
   return true;
 }
