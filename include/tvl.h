@@ -76,7 +76,7 @@ size_t tvl_blob_bytes(const tvl_config* cfg, int32_t tied);
  *              creates and owns a non-blocking stream.
  *   out        receives the handle (NULL on failure).
  * GPU-path requirements (else TVL_E_UNSUPPORTED): dim % 32 == 0,
- * head_dim % 4 == 0 and <= 256, hidden_dim % 4 == 0, max(dim, hidden_dim)
+ * head_dim % 4 == 0 and <= 128, hidden_dim % 4 == 0, max(dim, hidden_dim)
  * <= 16384. Invalid shapes give TVL_E_INVAL. Uses the current CUDA device. */
 tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, void* stream,
                     tvl_model** out);

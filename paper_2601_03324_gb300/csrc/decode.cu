@@ -43,9 +43,10 @@ SmemPlan plan_smem(int d, int F, int hd, int H, int nch_cap, int max_bytes) {
   SmemPlan p{};
   const int att_floats =
       std::max(3 * hd + kAttMaxChunk + 4 * kConsumerThreads, 2 * H * nch_cap) + 16;
+  // every region is a multiple of 128 bytes, so every region starts aligned
   const int xs = (int)a128(4LL * d), vec = (int)a128(4LL * std::max(d, F));
-  const int seg = kMaxSegParts * 4, att = (int)a128(4LL * att_floats), misc = 256;
-  const int bars = kRingBarBytes;
+  const int seg = (int)a128(kMaxSegParts * 4), att = (int)a128(4LL * att_floats), misc = 256;
+  const int bars = (int)a128(kRingBarBytes);
   const int other = bars + xs + vec + seg + att + misc;
   int nst = (max_bytes - other) / kStageBytes;
   if (nst > kMaxStages) nst = kMaxStages;
@@ -139,8 +140,8 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   }
   const int d = cfg->dim, F = cfg->hidden_dim, H = cfg->n_heads, Hkv = cfg->n_kv_heads;
   const int hd = d / H, kvd = Hkv * hd, V = cfg->vocab_size, S = cfg->max_seq, L = cfg->n_layers;
-  if (d % 32 != 0 || hd % 4 != 0 || hd > 256 || F % 4 != 0 || std::max(d, F) > 16384) {
-    set_error("tvl_load: the GPU path needs dim % 32 == 0, head_dim % 4 == 0 and <= 256, "
+  if (d % 32 != 0 || hd % 4 != 0 || hd > 128 || F % 4 != 0 || std::max(d, F) > 16384) {
+    set_error("tvl_load: the GPU path needs dim % 32 == 0, head_dim % 4 == 0 and <= 128, "
               "hidden_dim % 4 == 0, max(dim, hidden_dim) <= 16384");
     return TVL_E_UNSUPPORTED;
   }

@@ -201,7 +201,8 @@ extern "C" tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t
   a.nv = (long long)d_out * a.S;
   const int G = (int)(a.nv < info.sms ? a.nv : info.sms);
   // shared memory: ring | barriers | x | piece sums | misc
-  const int xbytes = (int)a128(4LL * d_in), segb = kMaxSegParts * 4, bars = kRingBarBytes;
+  const int xbytes = (int)a128(4LL * d_in), segb = (int)a128(kMaxSegParts * 4);
+  const int bars = (int)a128(kRingBarBytes);  // every region a 128-byte multiple
   const int misc = 128;
   int nst = (info.max_optin - xbytes - segb - bars - misc) / kStageBytes;
   if (nst > kMaxStages) nst = kMaxStages;

@@ -235,6 +235,26 @@ __device__ __forceinline__ float row_partial(const float4* w4, const float4* x4,
   return ((c0.x + c0.y) + (c0.z + c0.w)) + ((c1.x + c1.y) + (c1.z + c1.w));
 }
 
+// Two rows with the same columns in one pass: each x float4 is read once
+// for both (half the shared-memory traffic of two separate passes).
+__device__ __forceinline__ float2 row2_partial(const float4* w0, const float4* w1, const float4* x4,
+                                               int n4, int lane) {
+  float4 a = make_float4(0.f, 0.f, 0.f, 0.f), b = a;
+#pragma unroll 2
+  for (int e = lane; e < n4; e += 32) {
+    const float4 x = x4[e], u = w0[e], v = w1[e];
+    a.x = fmaf(u.x, x.x, a.x);
+    a.y = fmaf(u.y, x.y, a.y);
+    a.z = fmaf(u.z, x.z, a.z);
+    a.w = fmaf(u.w, x.w, a.w);
+    b.x = fmaf(v.x, x.x, b.x);
+    b.y = fmaf(v.y, x.y, b.y);
+    b.z = fmaf(v.z, x.z, b.z);
+    b.w = fmaf(v.w, x.w, b.w);
+  }
+  return make_float2((a.x + a.y) + (a.z + a.w), (b.x + b.y) + (b.z + b.w));
+}
+
 // Same for rows of at most 1024 floats with the lane's slice of x already in
 // registers: xr[k] holds x float4 lane + 32k.
 __device__ __forceinline__ float row_partial_xr(const float4* w4, const float4 (&xr)[8], int n4,
@@ -363,11 +383,15 @@ __device__ inline bool consume_phase(const Ring& r, uint32_t& g, const StagePlan
         if (two) a1 = row_partial_xr(w1, xr, n4, lane);
       } else {
         const float* xb = xs + s.c0;
-        a0 = row_partial(w0, reinterpret_cast<const float4*>(xb + (S > 1 ? (v0 % S) * Kc : 0)),
-                         n4, lane);
-        if (two)
-          a1 = row_partial(w1, reinterpret_cast<const float4*>(xb + (S > 1 ? (v1 % S) * Kc : 0)),
-                           n4, lane);
+        const int o0 = S > 1 ? (v0 % S) * Kc : 0, o1 = S > 1 ? (v1 % S) * Kc : 0;
+        if (two && o0 == o1) {  // same input columns: one pass for both rows
+          const float2 r2 = row2_partial(w0, w1, reinterpret_cast<const float4*>(xb + o0), n4, lane);
+          a0 = r2.x;
+          a1 = r2.y;
+        } else {
+          a0 = row_partial(w0, reinterpret_cast<const float4*>(xb + o0), n4, lane);
+          if (two) a1 = row_partial(w1, reinterpret_cast<const float4*>(xb + o1), n4, lane);
+        }
       }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
