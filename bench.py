@@ -78,23 +78,43 @@ def kernel_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def committed_traffic(workload: str):
-    """dram bytes per step from the committed ncu summary, if it was taken
-    on the kernel sources as they are now."""
+def committed_traffic(workload: str, bytes_launch: int):
+    """DRAM bytes of one launch of bytes_launch algorithmic bytes, from the
+    committed ncu summary, if it was taken on the kernel sources as they are
+    now. The capture covers a short launch; its read+write bytes are scaled by
+    the ratio of algorithmic bytes (the traffic follows the bytes streamed)."""
     p = os.path.join(ROOT, "profiles", f"decode_kernel_{workload}.txt")
     if not os.path.exists(p):
         return None
     kv = {}
     for line in open(p):
-        if ":" in line:
+        if ":" in line and not line.startswith("#"):
             k, v = line.split(":", 1)
             kv[k.strip()] = v.strip()
     if kv.get("kernel_sources_sha256_16") != kernel_hash():
         return None
     try:
-        return float(kv["dram_bytes_per_step"])
-    except (KeyError, ValueError):
+        dram = float(kv["dram_bytes_read"]) + float(kv["dram_bytes_write"])
+        return dram * bytes_launch / float(kv["captured_algorithmic_bytes"])
+    except (KeyError, ValueError, ZeroDivisionError):
         return None
+
+
+def max_over_ranks(x: float, world: int, device: str) -> float:
+    """The largest x over all ranks (the job's time is its slowest rank's)."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tokens_per_s(world: int, steps: int, max_ms: float) -> float:
+    """Whole-job throughput: every rank decodes `steps` tokens of its own
+    sequences (replicas), the job ends with its slowest rank."""
+    return world * steps / (max_ms * 1e-3)
 
 
 def step_bytes(cfg: dict, streamed: int, pos: int) -> int:
@@ -338,10 +358,7 @@ def main():
         dist.barrier()
     el_ms = start.elapsed_time(end)
     clk = clocks.stop(t_wall0, t_wall1)
-    el_t = torch.tensor([el_ms], device="cuda")
-    if world > 1:
-        dist.all_reduce(el_t, op=dist.ReduceOp.MAX)
-    el_ms = float(el_t.item())
+    el_ms = max_over_ranks(el_ms, world, "cuda")
 
     # per-launch roofline of the decode kernel (full-length launches)
     full = [(a.elapsed_time(b), n) for (a, b, n) in ev]
@@ -350,7 +367,7 @@ def main():
     bytes_launch = sum(step_bytes(cfg, info.streamed_bytes, p) for p in range(n_typ))
     peak, peak_src = measured_peaks()
     achieved = bytes_launch / (statistics.mean(t for t, n in full if n == n_typ) * 1e-3) / 1e9
-    traffic = committed_traffic(args.workload)
+    traffic = committed_traffic(args.workload, bytes_launch)
     steps_ns = model.step_times(n_typ).astype(np.float64)
     dts = np.diff(steps_ns) / 1e3 if n_typ > 1 else np.array([launch_ms * 1e3])
 
@@ -385,7 +402,7 @@ def main():
                "sample": f"first {n} greedy steps of the workload from token 1 "
                          f"({el:.1f} s, double accumulators, one thread)"}
 
-    value = world * args.steps / (el_ms * 1e-3)
+    value = job_tokens_per_s(world, args.steps, el_ms)
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": el_ms / args.steps,

@@ -1,0 +1,86 @@
+"""Host-side logic of bench.py on CPU: the multi-rank aggregation (gloo,
+world size 2) and the reference arm's rank handling. Replicas only: every rank
+decodes its own sequences, so the only collective is the timing reduction."""
+import argparse
+import json
+import os
+import socket
+import sys
+
+import pytest
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+
+def _free_port() -> int:
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, q):
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    sys.path.insert(0, ROOT)
+    import bench
+    dist.init_process_group("gloo", init_method="env://")
+    try:
+        env = bench.dist_env()
+        # rank r took (r + 1) * 100 ms for its steps
+        ms = bench.max_over_ranks(100.0 * (rank + 1), world, "cpu")
+        q.put((rank, env, ms, bench.job_tokens_per_s(world, 512, ms)))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_max_over_ranks_gloo_world2():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_main, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    out = sorted(q.get(timeout=120) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    for rank, env, ms, val in out:
+        assert env == (rank, rank, 2)
+        assert ms == 200.0                      # the slowest rank's time, on every rank
+        assert val == pytest.approx(2 * 512 / 0.2)  # all ranks' tokens / max time
+
+
+def test_single_rank_needs_no_process_group():
+    import bench
+    assert bench.max_over_ranks(3.5, 1, "cpu") == 3.5
+    assert bench.job_tokens_per_s(1, 100, 50.0) == pytest.approx(2000.0)
+
+
+def _ref_args(**kw):
+    a = dict(gpus=2, steps=1, warmup=0, impl="reference", workload="tiny", no_e2e=False,
+             no_cpu_baseline=False, cpu_seconds=1.0, gemv_sweep=False)
+    a.update(kw)
+    return argparse.Namespace(**a)
+
+
+def test_reference_arm_other_ranks_exit_without_work(capsys):
+    import bench
+    from paper_2601_03324_gb300 import synth
+    cfg = synth.model_config("tiny")
+    assert bench.run_reference(_ref_args(), cfg, rank=1, world=2) == 0
+    assert capsys.readouterr().out == ""
+
+
+def test_reference_arm_rank0_line(capsys):
+    import bench
+    from paper_2601_03324_gb300 import synth
+    cfg = synth.model_config("tiny")
+    assert bench.run_reference(_ref_args(), cfg, rank=0, world=2) == 0
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["n_gpus"] == 2
+    assert line["value"] > 0 and line["unit"] == "tokens/s" and line["higher_is_better"]
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 1
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
