@@ -119,6 +119,27 @@ tvl_status tvl_decode_greedy(tvl_model* m, int32_t start_token, int32_t start_po
 tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t d_out, int32_t d_in,
                     void* stream);
 
+/* tvl_gemv without any allocation. The paper has no counterpart: this entry
+ * exists for callers that cannot allocate device memory at call time — a host
+ * thread that must not stall other streams (cudaMalloc and cudaFree may
+ * synchronise the device implicitly), or a caller that has handed all device
+ * memory to its own pool (tvl_gemv's first short-and-wide call on a stream
+ * allocates its scratch and could fail there).
+ * Same arguments, layout, paths and results as tvl_gemv (same kernel, same
+ * split, bit-identical output). The split-K scratch is one static module
+ * array of 48 KB per device (8192 partials, 4096 row counters), not
+ * allocated memory. A shape whose split needs more (never on a 152-SM GB300:
+ * at most 4864 partials and 2431 rows) returns TVL_E_UNSUPPORTED with the
+ * sizes in tvl_last_error(); use tvl_gemv for it.
+ * The FIRST call on a device does a one-time setup: it looks up the array's
+ * device address, zeroes its counters on `stream` and waits for that, so make
+ * it before any work that must not wait (e.g. before a stream capture).
+ * The scratch is shared by every call on the device: calls that can overlap
+ * on the device (different streams without ordering between them) race on it
+ * and give wrong results; order them, or use tvl_gemv. */
+tvl_status tvl_gemv_noalloc(const float* W, const float* x, float* y, int32_t d_out,
+                            int32_t d_in, void* stream);
+
 /* Wait for the model's queued work, then report any device-side error. */
 tvl_status tvl_sync(tvl_model* m);
 

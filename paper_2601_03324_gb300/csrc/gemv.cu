@@ -9,6 +9,7 @@
 // counter). The result does not depend on timing. Every wait in the kernel is
 // bounded (one second); a CTA whose stage never lands leaves early, which
 // only a broken device can cause.
+#include <cstdio>
 #include <map>
 #include <mutex>
 #include <utility>
@@ -240,6 +241,124 @@ extern "C" tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t
     a.part = ws.part;
     a.cnt = ws.cnt;
   }
+  TVL_CK(cudaFuncSetAttribute((const void*)gemv_stream_kernel,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+  gemv_stream_kernel<<<G, kThreads, smem, s>>>(a);
+  TVL_CK(cudaGetLastError());
+  return TVL_OK;
+}
+
+// ---- tvl_gemv_noalloc: the same GEMV with its split-K scratch in module memory ----
+
+namespace {
+
+// Split-K partials (floats) and per-row arrival counters (ints) of
+// tvl_gemv_noalloc. split_for keeps M * S below 32 x the SM count and M below
+// 16 x the SM count whenever S > 1, so on a 152-SM part at most 4864 partials
+// and 2431 counters are live; the sizes below leave room for larger parts.
+constexpr int kNoAllocPart = 8192;
+constexpr int kNoAllocRows = 4096;
+constexpr size_t kNoAllocBytes = 4 * (size_t)kNoAllocPart + 4 * (size_t)kNoAllocRows;  // 48 KB
+static __device__ __align__(256) unsigned char g_gemv_scratch[kNoAllocBytes];
+
+constexpr int kNoAllocMaxDevices = 64;
+struct NoAllocDev {
+  bool ready;
+  int sms, max_optin;
+  float* part;
+  int* cnt;
+};
+NoAllocDev g_noalloc[kNoAllocMaxDevices];  // fixed table: no heap use on any call
+std::mutex g_noalloc_mu;
+
+}  // namespace
+
+extern "C" tvl_status tvl_gemv_noalloc(const float* W, const float* x, float* y, int32_t d_out,
+                                       int32_t d_in, void* stream) {
+  if (!W || !x || !y || d_out < 1 || d_in < 1) {
+    set_error("tvl_gemv_noalloc: null pointer or non-positive size");
+    return TVL_E_INVAL;
+  }
+  cudaStream_t s = (cudaStream_t)stream;
+  int dev = 0;
+  TVL_CK(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kNoAllocMaxDevices) {
+    char msg[128];
+    snprintf(msg, sizeof msg, "tvl_gemv_noalloc: device ordinal %d is beyond the %d-entry table",
+             dev, kNoAllocMaxDevices);
+    set_error(msg);
+    return TVL_E_UNSUPPORTED;
+  }
+  NoAllocDev nd;
+  {
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    NoAllocDev& e = g_noalloc[dev];
+    if (!e.ready) {  // once per device: address of the module array, counters to zero
+      void* base = nullptr;
+      TVL_CK(cudaGetSymbolAddress(&base, g_gemv_scratch));
+      TVL_CK(cudaDeviceGetAttribute(&e.sms, cudaDevAttrMultiProcessorCount, dev));
+      TVL_CK(cudaDeviceGetAttribute(&e.max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev));
+      e.part = reinterpret_cast<float*>(base);
+      e.cnt = reinterpret_cast<int*>(reinterpret_cast<unsigned char*>(base) + 4 * (size_t)kNoAllocPart);
+      TVL_CK(cudaMemsetAsync(e.cnt, 0, 4 * (size_t)kNoAllocRows, s));
+      TVL_CK(cudaStreamSynchronize(s));
+      e.ready = true;
+    }
+    nd = e;
+  }
+  const bool aligned = ((uintptr_t)W % 16 == 0) && ((uintptr_t)x % 16 == 0) && d_in % 4 == 0;
+  bool fits = aligned && d_in <= 16384;
+  const int S = fits ? split_for(d_out, d_in, nd.sms) : 1;
+  const long long nv = (long long)d_out * S;
+  if (fits) {  // segment partials of rows longer than a stage must fit the shared scratch
+    const long long G = nv < nd.sms ? nv : nd.sms;
+    const StagePlan pl = plan_stages(nv, d_in / S, (int)G, 0);
+    fits = pl.spr == 1 || ((nv + G - 1) / G) * pl.spr <= kMaxSegParts;
+  }
+  if (!fits) {
+    const int threads = 256, rows_per_block = threads / 32;
+    gemv_rowwise_kernel<<<(d_out + rows_per_block - 1) / rows_per_block, threads, 0, s>>>(
+        W, x, y, d_out, d_in);
+    TVL_CK(cudaGetLastError());
+    return TVL_OK;
+  }
+  if (S > 1 && (nv > kNoAllocPart || d_out > kNoAllocRows)) {
+    char msg[192];
+    snprintf(msg, sizeof msg,
+             "tvl_gemv_noalloc: %d x %d splits into %lld partials over %d rows; the static "
+             "scratch holds %d partials and %d rows (use tvl_gemv)",
+             (int)d_out, (int)d_in, nv, (int)d_out, kNoAllocPart, kNoAllocRows);
+    set_error(msg);
+    return TVL_E_UNSUPPORTED;
+  }
+  GemvArgs a{};
+  a.W = W;
+  a.x = x;
+  a.y = y;
+  a.M = d_out;
+  a.K = d_in;
+  a.S = S;
+  a.Kc = d_in / S;
+  a.nv = nv;
+  a.part = nd.part;
+  a.cnt = nd.cnt;
+  const int G = (int)(nv < nd.sms ? nv : nd.sms);
+  const int xbytes = (int)a128(4LL * d_in), segb = (int)a128(kMaxSegParts * 4);
+  const int bars = (int)a128(kRingBarBytes);
+  const int misc = 128;
+  int nst = (nd.max_optin - xbytes - segb - bars - misc) / kStageBytes;
+  if (nst > kMaxStages) nst = kMaxStages;
+  if (nst < 2) {
+    set_error("tvl_gemv_noalloc: not enough shared memory");
+    return TVL_E_UNSUPPORTED;
+  }
+  a.nst = nst;
+  a.sm_ring = 0;
+  a.sm_bars = nst * kStageBytes;
+  a.sm_x = a.sm_bars + bars;
+  a.sm_seg = a.sm_x + xbytes;
+  a.sm_misc = a.sm_seg + segb;
+  const int smem = a.sm_misc + misc;
   TVL_CK(cudaFuncSetAttribute((const void*)gemv_stream_kernel,
                               cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
   gemv_stream_kernel<<<G, kThreads, smem, s>>>(a);

@@ -64,6 +64,8 @@ def _load():
     L.tvl_decode_greedy.argtypes = [P, i32, i32, i32, P]
     L.tvl_gemv.restype = st
     L.tvl_gemv.argtypes = [P, P, P, i32, i32, P]
+    L.tvl_gemv_noalloc.restype = st
+    L.tvl_gemv_noalloc.argtypes = [P, P, P, i32, i32, P]
     L.tvl_sync.restype = st
     L.tvl_sync.argtypes = [P]
     L.tvl_free.restype = None
@@ -84,7 +86,7 @@ def _load():
 lib = _load()
 
 EXPORTED = ["tvl_blob_bytes", "tvl_load", "tvl_load_file", "tvl_forward", "tvl_decode_greedy",
-            "tvl_gemv", "tvl_sync", "tvl_free", "tvl_status_string", "tvl_last_error",
+            "tvl_gemv", "tvl_gemv_noalloc", "tvl_sync", "tvl_free", "tvl_status_string", "tvl_last_error",
             "tvl_get_info", "tvl_step_times", "tvl_selftest_barrier_timeout"]
 
 
@@ -127,6 +129,13 @@ def tvl_gemv(W, x, y, d_out: int, d_in: int, stream: int = 0):
     _check(lib.tvl_gemv(ctypes.c_void_p(_addr(W)), ctypes.c_void_p(_addr(x)),
                         ctypes.c_void_p(_addr(y)), int(d_out), int(d_in),
                         ctypes.c_void_p(int(stream))), "tvl_gemv")
+
+
+def tvl_gemv_noalloc(W, x, y, d_out: int, d_in: int, stream: int = 0):
+    """tvl_gemv with its scratch in a static module array (nothing allocated)."""
+    _check(lib.tvl_gemv_noalloc(ctypes.c_void_p(_addr(W)), ctypes.c_void_p(_addr(x)),
+                                ctypes.c_void_p(_addr(y)), int(d_out), int(d_in),
+                                ctypes.c_void_p(int(stream))), "tvl_gemv_noalloc")
 
 
 def tvl_selftest_barrier_timeout(limit_ms: int) -> int:
