@@ -640,39 +640,42 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
     for (int j = tid; j < (a.d >> 2); j += kConsumerThreads)
       reinterpret_cast<float4*>(xs)[j] = __ldg(e4 + j);
     named_bar_sync(kBarConsumers, kConsumerThreads);
+    // The four GEMV phases of a layer run one copy of the phase code, in a
+    // loop that is not unrolled, so the code stays in the instruction cache
+    // from one phase to the next. Phase k's prologue leaves its input in vec.
     for (int l = 0; l < a.L; ++l) {
       const unsigned char* lw = a.layer0 + (size_t)l * a.layer_stride;
       const unsigned el = es + (unsigned)(kPhasesPerLayer * l);
-      if (l > 0 && !add_published(a.x_f, el - 1)) return false;
-      rmsnorm_to(vec, xs, reinterpret_cast<const float*>(lw + a.o_gatt), a.d, a.eps, red);
-      EpiTag e_qkv{a.x_qkv, el};
-      if (!consume_phase<false>(r, g, plan_stages(a.d + 2 * a.kvd, a.d, a.G, c), vec, 1, a.d, seg,
-                         e_qkv, a.err, a.err_host, s_abort))
-        return false;
-      if (!attention_phase(a, l, pos, el, el + 1, asm_, red, pc)) return false;
-      if (!merge_attention(a, pos, el + 1, vec, asm_, pc)) return false;
-      EpiTag e_o{a.x_o, el + 2};
-      if (!consume_phase<false>(r, g, plan_stages(a.d, a.d, a.G, c), vec, 1, a.d, seg, e_o, a.err,
-                         a.err_host, s_abort))
-        return false;
-      if (!add_published(a.x_o, el + 2)) return false;
-      rmsnorm_to(vec, xs, reinterpret_cast<const float*>(lw + a.o_gffn), a.d, a.eps, red);
-      EpiTag e_13{a.x_h13, el + 3};
-      if (!consume_phase<false>(r, g, plan_stages(2 * a.F, a.d, a.G, c), vec, 1, a.d, seg, e_13, a.err,
-                         a.err_host, s_abort))
-        return false;
-      {  // h = silu(a) * b (paper §2.1, SwiGLU); a = h13[k], b = h13[F + k]
-        const bool ok = poll_pairs2(a.x_h13, a.x_h13 + a.F, a.F >> 1, el + 3, pc,
-                                    [&](int p, float a0, float a1, float b0, float b1) {
-                                      vec[2 * p] = (a0 / (1.0f + expf(-a0))) * b0;
-                                      vec[2 * p + 1] = (a1 / (1.0f + expf(-a1))) * b1;
-                                    });
-        if (!vote_ok(ok, s_abort)) return false;
+#pragma unroll 1
+      for (int k = 0; k < 4; ++k) {
+        if (k == 0 || k == 2) {
+          // x += (the previous phase's published output), then x_b = RMSNorm(x, g)
+          if (k == 2 || l > 0) {
+            if (!add_published(k == 0 ? a.x_f : a.x_o, k == 0 ? el - 1 : el + 2)) return false;
+          }
+          rmsnorm_to(vec, xs, reinterpret_cast<const float*>(lw + (k == 0 ? a.o_gatt : a.o_gffn)),
+                     a.d, a.eps, red);
+        } else if (k == 1) {
+          if (!attention_phase(a, l, pos, el, el + 1, asm_, red, pc)) return false;
+          if (!merge_attention(a, pos, el + 1, vec, asm_, pc)) return false;
+        } else {  // h = silu(a) * b (paper §2.1, SwiGLU); a = h13[i], b = h13[F + i]
+          const bool ok = poll_pairs2(a.x_h13, a.x_h13 + a.F, a.F >> 1, el + 3, pc,
+                                      [&](int p, float a0, float a1, float b0, float b1) {
+                                        vec[2 * p] = (a0 / (1.0f + expf(-a0))) * b0;
+                                        vec[2 * p + 1] = (a1 / (1.0f + expf(-a1))) * b1;
+                                      });
+          if (!vote_ok(ok, s_abort)) return false;
+        }
+        // [Wq|Wk|Wv] x_b, Wo o, [W1|W3] x_b, W2 h: M rows of K columns, published
+        // with the exchange tag of phase k (the attention partials take el + 1)
+        const int M = k == 0 ? a.d + 2 * a.kvd : k == 2 ? 2 * a.F : a.d;
+        const int K = k == 3 ? a.F : a.d;
+        unsigned long long* out = k == 0 ? a.x_qkv : k == 1 ? a.x_o : k == 2 ? a.x_h13 : a.x_f;
+        EpiTag e{out, el + (k == 0 ? 0u : (unsigned)k + 1u)};
+        if (!consume_phase<false>(r, g, plan_stages(M, K, a.G, c), vec, 1, K, seg, e, a.err,
+                                  a.err_host, s_abort))
+          return false;
       }
-      EpiTag e_2{a.x_f, el + 4};
-      if (!consume_phase<false>(r, g, plan_stages(a.d, a.F, a.G, c), vec, 1, a.F, seg, e_2, a.err,
-                         a.err_host, s_abort))
-        return false;
     }
     if (a.L > 0 && !add_published(a.x_f, es + per_step - 2)) return false;
     rmsnorm_to(vec, xs, a.g_final, a.d, a.eps, red);
