@@ -362,6 +362,25 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
     const int t0 = c * clen;
     const int t1 = (t0 + clen < pos + 1) ? t0 + clen : pos + 1;
     const bool has_new = (t1 == pos + 1);
+    const float* kbase = a.kc + lay + kvh * hd;
+    const float* vbase = a.vc + lay + kvh * hd;
+    const int pstride = kConsumerWarps * ppw;
+    const int ng = kConsumerThreads / hd4;
+    const int gi = tid / hd4, f = tid - gi * hd4;
+    const int n = t1 - t0;
+    const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
+    float4 kr0 = z4, kr1 = z4, v0 = z4, v1 = z4;
+    {
+      const int tk = t0 + warp * ppw + sub;
+      if (li < hd4 && tk < t1 && tk != pos)
+        kr0 = ldcg4(reinterpret_cast<const float4*>(kbase + (size_t)tk * a.kvd) + li);
+      if (li < hd4 && tk + pstride < t1 && tk + pstride != pos)
+        kr1 = ldcg4(reinterpret_cast<const float4*>(kbase + (size_t)(tk + pstride) * a.kvd) + li);
+      if (gi < ng && gi < n && t0 + gi != pos)
+        v0 = ldcg4(reinterpret_cast<const float4*>(vbase + (size_t)(t0 + gi) * a.kvd) + f);
+      if (gi < ng && gi + ng < n && t0 + gi + ng != pos)
+        v1 = ldcg4(reinterpret_cast<const float4*>(vbase + (size_t)(t0 + gi + ng) * a.kvd) + f);
+    }
     // q (and the new k, v) with RoPE: pair i turns by pos * theta^(-2i/hd).
     // Pair i of a head is one 16-byte tagged load.
     const int nget = has_new ? 3 * half : half;
@@ -384,7 +403,6 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
       }
     }
     if (!vote_ok(ok, pc.s_abort)) return false;
-    __threadfence();  // the K/V rows below were published by other CTAs' earlier steps
     if (has_new && (h % group) == 0) {  // one writer per kv head
       float* kd = a.kc + lay + (size_t)pos * a.kvd + kvh * hd;
       float* vd = a.vc + lay + (size_t)pos * a.kvd + kvh * hd;
@@ -392,12 +410,13 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
         kd[j] = kp[j];
         vd[j] = vp[j];
       }
-      __threadfence();  // cache row visible before this item's partials are
+      if (tid < hd) __threadfence();  // cache row visible before this item's partials are
     }
-    // scores s_t = (q . k_t) * scale for t in [t0, t1), two passes of loads in flight
+    if (gi < ng && t0 + gi == pos) v0 = reinterpret_cast<const float4*>(vp)[f];
+    if (gi < ng && t0 + gi + ng == pos) v1 = reinterpret_cast<const float4*>(vp)[f];
+    // scores s_t = (q . k_t) * scale for t in [t0, t1); the first pass uses the rows loaded above
     const float4* q4 = reinterpret_cast<const float4*>(q);
-    const int pstride = kConsumerWarps * ppw;
-    for (int tb = t0 + warp * ppw; tb < t1; tb += 2 * pstride) {
+    for (int tb = t0 + warp * ppw, first = 1; tb < t1; tb += 2 * pstride, first = 0) {
       float acc[2] = {0.f, 0.f};
 #pragma unroll
       for (int u = 0; u < 2; ++u) {
@@ -405,10 +424,9 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
         if (t < t1) {
           const float4* k4 = (t == pos)
                                  ? reinterpret_cast<const float4*>(kp)
-                                 : reinterpret_cast<const float4*>(a.kc + lay + (size_t)t * a.kvd +
-                                                                   kvh * hd);
+                                 : reinterpret_cast<const float4*>(kbase + (size_t)t * a.kvd);
           for (int f = li; f < hd4; f += lpp) {
-            const float4 kv = (t == pos) ? k4[f] : ldcg4(k4 + f);
+            const float4 kv = (t == pos) ? k4[f] : first ? (u ? kr1 : kr0) : ldcg4(k4 + f);
             const float4 qv = q4[f];
             acc[u] = fmaf(qv.x, kv.x, acc[u]);
             acc[u] = fmaf(qv.y, kv.y, acc[u]);
@@ -425,18 +443,11 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
         if (t < t1 && li == 0) sc[t - t0] = s * a.att_scale;
       }
     }
-    // V rows of the first positions of this thread, loaded while the softmax runs
-    const int ng = kConsumerThreads / hd4;
-    const int gi = tid / hd4, f = tid - gi * hd4;
-    const int n = t1 - t0;
     auto vrow = [&](int t) -> float4 {
       return (t == pos) ? reinterpret_cast<const float4*>(vp)[f]
                         : ldcg4(reinterpret_cast<const float4*>(a.vc + lay + (size_t)t * a.kvd +
                                                                 kvh * hd) + f);
     };
-    float4 v0 = make_float4(0.f, 0.f, 0.f, 0.f), v1 = v0;
-    if (gi < ng && gi < n) v0 = vrow(t0 + gi);
-    if (gi < ng && gi + ng < n) v1 = vrow(t0 + gi + ng);
     named_bar_sync(kBarConsumers, kConsumerThreads);
     float m = -INFINITY;
     for (int i = tid; i < n; i += kConsumerThreads) m = fmaxf(m, sc[i]);
@@ -635,6 +646,10 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
         a.ts[s - 1] = globaltimer_ns();
       }
     }
+    // Acquire: K/V rows written in earlier steps were released (fence, then a
+    // published record) before this CTA read those records; this fence and the
+    // barrier below order every later row load of the CTA after them.
+    if (tid == 0) __threadfence();
     // x = E[token] (paper §4.1: weights are rows at offsets in the blob)
     const float4* e4 = reinterpret_cast<const float4*>(a.E + (size_t)token * a.d);
     for (int j = tid; j < (a.d >> 2); j += kConsumerThreads)
