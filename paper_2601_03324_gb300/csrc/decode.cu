@@ -41,8 +41,7 @@ struct SmemPlan {
 
 SmemPlan plan_smem(int d, int F, int hd, int H, int nch_cap, int max_bytes) {
   SmemPlan p{};
-  const int att_floats =
-      std::max(3 * hd + kAttMaxChunk + 4 * kConsumerThreads, 2 * H * nch_cap) + 16;
+  const int att_floats = 3 * hd + kAttMaxChunk + 4 * kConsumerThreads + nch_cap * (hd + 2) + 16;
   // every region is a multiple of 128 bytes, so every region starts aligned
   const int xs = (int)a128(4LL * d), vec = (int)a128(4LL * std::max(d, F));
   const int seg = (int)a128(kMaxSegParts * 4), att = (int)a128(4LL * att_floats), misc = 256;
@@ -235,6 +234,7 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   const size_t o_qkv = take(8ull * (d + 2 * kvd)), o_o = take(8ull * d), o_h13 = take(16ull * F);
   const size_t o_f = take(8ull * d), o_lg = take(4ull * V);
   const size_t o_att = take(8ull * H * nch_cap * att_stride);
+  const size_t o_attn = take(8ull * d);
   const size_t o_cand = take(8ull * 2 * G * 2), o_tok = take(4ull * S);
   const size_t o_ts = take(8ull * S), o_err = take(4);
   m->arena_bytes = off;
@@ -328,6 +328,7 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   a.x_f = reinterpret_cast<unsigned long long*>(m->arena + o_f);
   a.logits = reinterpret_cast<float*>(m->arena + o_lg);
   a.x_att = reinterpret_cast<unsigned long long*>(m->arena + o_att);
+  a.x_attn = reinterpret_cast<unsigned long long*>(m->arena + o_attn);
   a.x_cand = reinterpret_cast<unsigned long long*>(m->arena + o_cand);
   a.tokens = reinterpret_cast<int*>(m->arena + o_tok);
   a.ts = reinterpret_cast<unsigned long long*>(m->arena + o_ts);

@@ -48,7 +48,8 @@ struct DecodeArgs {
   float* vc;
   // tagged exchange buffers (64-bit words: tag << 32 | float bits)
   unsigned long long* x_qkv;   // [d + 2 kvd]
-  unsigned long long* x_att;   // [H][nch_cap][att_stride]: m, l, -, -, o[hd]
+  unsigned long long* x_att;   // [H][nch_cap][att_stride]: m, l, -, -, sum[hd] of chunks > 0
+  unsigned long long* x_attn;  // [d]: attention output, merged per head
   unsigned long long* x_o;     // [d]
   unsigned long long* x_h13;   // [2F]
   unsigned long long* x_f;     // [d]
@@ -212,6 +213,41 @@ __device__ inline bool poll_pairs2(const unsigned long long* sa, const unsigned 
   return true;
 }
 
+// Poll pairs p = tid, tid + 224, ... (npairs pairs) at addresses addr(p), up
+// to four 16-byte loads in flight per thread; fn(p, v0, v1) takes each ready
+// pair. Returns false if this thread gave up (the caller votes).
+template <class Addr, class Fn>
+__device__ inline bool poll_pairs_at(int npairs, Addr addr, unsigned tag, const Poll& c, Fn fn) {
+  for (int base = threadIdx.x; base < npairs; base += kConsumerThreads * 4) {
+    ulonglong2 v[4];
+    unsigned pending = 0;
+#pragma unroll
+    for (int b = 0; b < 4; ++b) {
+      const int p = base + b * kConsumerThreads;
+      if (p < npairs) {
+        v[b] = ld_tag2(addr(p));
+        pending |= 1u << b;
+      }
+    }
+    PollClock clk;
+    while (true) {
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        if (((pending >> b) & 1u) && tags_are(v[b], tag)) {
+          fn(base + b * kConsumerThreads, lo_f(v[b].x), lo_f(v[b].y));
+          pending &= ~(1u << b);
+        }
+      }
+      if (!pending) break;
+      if (!clk.keep_waiting(c)) return false;
+#pragma unroll
+      for (int b = 0; b < 4; ++b)
+        if ((pending >> b) & 1u) v[b] = ld_tag2(addr(base + b * kConsumerThreads));
+    }
+  }
+  return true;
+}
+
 // One pair, re-read until current (used where a thread needs a single pair).
 __device__ inline bool poll_one(const unsigned long long* p, unsigned tag, const Poll& c,
                                 ulonglong2& v) {
@@ -282,22 +318,27 @@ __device__ inline void block_argmax(float& v, int& idx, float* redv, int* redi) 
   named_bar_sync(kBarConsumers, kConsumerThreads);
 }
 
-// out = RMSNorm(x, g) (paper §11.2: ss/n + eps, 1/sqrt, then (x*g)*r). The
-// gain loads are issued before the reduction so that their latency overlaps it.
-__device__ inline void rmsnorm_to(float* out, const float* x, const float* g, int n, float eps,
-                                  float* red) {
-  const int n4 = n >> 2;
-  const float4* g4 = reinterpret_cast<const float4*>(g);
-  float4 gp[4];
+// RMSNorm gains, loaded into registers ahead of use so that their loads
+// overlap the exchange that delivers x (elements 4j..4j+3 for j = tid + 224k).
+struct Gains {
+  float4 v[4];
+  __device__ __forceinline__ void load(const float* g, int n) {
+    const float4* g4 = reinterpret_cast<const float4*>(g);
 #pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    const int j = threadIdx.x + k * kConsumerThreads;
-    if (j < n4) gp[k] = __ldg(g4 + j);
+    for (int k = 0; k < 4; ++k) {
+      const int j = threadIdx.x + k * kConsumerThreads;
+      if (j < (n >> 2)) v[k] = __ldg(g4 + j);
+    }
   }
-  float ss = 0.f;
-  for (int j = threadIdx.x; j < n; j += kConsumerThreads) ss = fmaf(x[j], x[j], ss);
-  const float tot = block_sum(ss, red);
+};
+
+// out = RMSNorm(x, g) (paper §11.2: ss/n + eps, 1/sqrt, then (x*g)*r), given
+// ss = this thread's share of the sum of x^2 and the preloaded gains.
+__device__ inline void rmsnorm_finish(float* out, const float* x, const Gains& gp, const float* g,
+                                      int n, float eps, float ss, float* red) {
+  const float tot = block_sum(ss, red);  // its barriers also publish x
   const float r = 1.0f / sqrtf(tot / (float)n + eps);
+  const int n4 = n >> 2;
   const float4* x4 = reinterpret_cast<const float4*>(x);
   float4* o4 = reinterpret_cast<float4*>(out);
   auto emit = [&](int j, const float4& gv) {
@@ -308,11 +349,18 @@ __device__ inline void rmsnorm_to(float* out, const float* x, const float* g, in
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
     const int j = threadIdx.x + k * kConsumerThreads;
-    if (j < n4) emit(j, gp[k]);
+    if (j < n4) emit(j, gp.v[k]);
   }
   for (int j = threadIdx.x + 4 * kConsumerThreads; j < n4; j += kConsumerThreads)
-    emit(j, __ldg(g4 + j));
+    emit(j, __ldg(reinterpret_cast<const float4*>(g) + j));
   named_bar_sync(kBarConsumers, kConsumerThreads);
+}
+
+// This thread's share of sum x^2 when no exchange delivered x.
+__device__ inline float sum_sq(const float* x, int n) {
+  float ss = 0.f;
+  for (int j = threadIdx.x; j < n; j += kConsumerThreads) ss = fmaf(x[j], x[j], ss);
+  return ss;
 }
 
 struct EpiTag {
@@ -356,8 +404,10 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
   const int ppw = 32 / lpp;
   const int sub = lane / lpp, li = lane - sub * lpp;
 
+  for (int pass = 0; pass < 2; ++pass)
   for (int it = blockIdx.x; it < a.H * nch; it += a.G) {
     const int h = it / nch, c = it - h * nch;
+    if ((c == 0) != (pass == 1)) continue;
     const int kvh = h / group;
     const int t0 = c * clen;
     const int t1 = (t0 + clen < pos + 1) ? t0 + clen : pos + 1;
@@ -474,89 +524,50 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
       reinterpret_cast<float4*>(part)[gi * hd4 + f] = acc;
     }
     named_bar_sync(kBarConsumers, kConsumerThreads);
-    unsigned long long* rec = a.x_att + ((size_t)h * a.nch_cap + c) * a.att_stride;
-    for (int j = tid; j < hd; j += kConsumerThreads) {
-      float o = 0.f;
-      for (int g2 = 0; g2 < ng; ++g2) o += part[g2 * hd + j];
-      st_tag(rec + 4 + j, tag_att, o);
-    }
-    if (tid == 0) {
-      st_tag(rec, tag_att, m);
-      st_tag(rec + 1, tag_att, ls);
+    float own = 0.f;  // this chunk's sum of e_t v_t, element tid (tid < hd)
+    if (tid < hd)
+      for (int g2 = 0; g2 < ng; ++g2) own += part[g2 * hd + tid];
+    if (c != 0) {
+      unsigned long long* rec = a.x_att + ((size_t)h * a.nch_cap + c) * a.att_stride;
+      if (tid < hd) st_tag(rec + 4 + tid, tag_att, own);
+      if (tid == 0) {
+        st_tag(rec, tag_att, m);
+        st_tag(rec + 1, tag_att, ls);
+      }
+    } else {
+      // the head's merger: records of chunks 1..nch-1 as pairs (m, l), (sum[2i], sum[2i+1]);
+      // o_h[j] = sum_c w_c sum_c[j], w_c = exp(m_c - M) / sum_c' exp(m_c' - M) l_c', chunk order
+      float* mrg = part + 4 * kConsumerThreads;  // [nch - 1][hd + 2]
+      const int ppr = 1 + half;
+      const bool ok2 = poll_pairs_at(
+          (nch - 1) * ppr,
+          [&](int p) {
+            const int cc = 1 + p / ppr, k = p - (cc - 1) * ppr;
+            const unsigned long long* r0 = a.x_att + ((size_t)h * a.nch_cap + cc) * a.att_stride;
+            return k == 0 ? r0 : r0 + 4 + 2 * (k - 1);
+          },
+          tag_att, pc, [&](int p, float x0, float x1) {
+            const int cc = p / ppr, k = p - cc * ppr;
+            float* rr = mrg + cc * (hd + 2);
+            rr[k == 0 ? 0 : 2 * k] = x0;
+            rr[k == 0 ? 1 : 2 * k + 1] = x1;
+          });
+      if (!vote_ok(ok2, pc.s_abort)) return false;
+      if (tid < hd) {
+        float M = m;
+        for (int cc = 0; cc < nch - 1; ++cc) M = fmaxf(M, mrg[cc * (hd + 2)]);
+        float Lsum = expf(m - M) * ls;
+        for (int cc = 0; cc < nch - 1; ++cc)
+          Lsum += expf(mrg[cc * (hd + 2)] - M) * mrg[cc * (hd + 2) + 1];
+        float o = (expf(m - M) / Lsum) * own;
+        for (int cc = 0; cc < nch - 1; ++cc)
+          o = fmaf(expf(mrg[cc * (hd + 2)] - M) / Lsum, mrg[cc * (hd + 2) + 2 + tid], o);
+        st_tag(a.x_attn + h * hd + tid, tag_att, o);
+      }
     }
     named_bar_sync(kBarConsumers, kConsumerThreads);
   }
   return true;
-}
-
-// o[h*hd + j] = sum_c w_c o_c[j] with w_c = exp(m_c - M) / sum_c exp(m_c - M) l_c.
-__device__ inline bool merge_attention(const DecodeArgs& a, int pos, unsigned tag, float* o,
-                                       float* sm, const Poll& pc) {
-  const int tid = threadIdx.x;
-  int nch, clen;
-  att_split(pos, a.H, a.G, &nch, &clen);
-  const int nrec = a.H * nch;
-  float* mv = sm;         // [H * nch]
-  float* wv = sm + nrec;  // [H * nch]
-  bool ok = true;
-  for (int i = tid; i < nrec && ok; i += kConsumerThreads) {
-    const int h = i / nch, c = i - h * nch;
-    const unsigned long long* src = a.x_att + ((size_t)h * a.nch_cap + c) * a.att_stride;
-    ulonglong2 v;
-    ok = poll_one(src, tag, pc, v);
-    mv[i] = lo_f(v.x);
-    wv[i] = lo_f(v.y);
-  }
-  if (!vote_ok(ok, pc.s_abort)) return false;
-  for (int h = tid; h < a.H; h += kConsumerThreads) {
-    float M = -INFINITY;
-    for (int c = 0; c < nch; ++c) M = fmaxf(M, mv[h * nch + c]);
-    float Lsum = 0.f;
-    for (int c = 0; c < nch; ++c) Lsum += expf(mv[h * nch + c] - M) * wv[h * nch + c];
-    for (int c = 0; c < nch; ++c) wv[h * nch + c] = expf(mv[h * nch + c] - M) / Lsum;
-  }
-  named_bar_sync(kBarConsumers, kConsumerThreads);
-  // output pairs (2p, 2p+1) of head h = 2p / hd: one 16-byte load per chunk,
-  // up to eight chunks in flight, re-read together until current
-  const int half = a.hd >> 1;
-  for (int p = tid; p < (a.d >> 1) && ok; p += kConsumerThreads) {
-    const int h = p / half, jp = p - h * half;
-    const unsigned long long* rec0 = a.x_att + (size_t)h * a.nch_cap * a.att_stride + 4 + 2 * jp;
-    float s0 = 0.f, s1 = 0.f;
-    for (int cb = 0; cb < nch && ok; cb += 8) {
-      const int ce = (nch - cb < 8) ? nch - cb : 8;
-      ulonglong2 v[8];
-      unsigned pending = 0;
-#pragma unroll
-      for (int k = 0; k < 8; ++k)
-        if (k < ce) {
-          v[k] = ld_tag2(rec0 + (size_t)(cb + k) * a.att_stride);
-          pending |= 1u << k;
-        }
-      PollClock clk;
-      while (ok) {
-#pragma unroll
-        for (int k = 0; k < 8; ++k)
-          if (((pending >> k) & 1u) && tags_are(v[k], tag)) pending &= ~(1u << k);
-        if (!pending) break;
-        ok = clk.keep_waiting(pc);
-#pragma unroll
-        for (int k = 0; k < 8; ++k)
-          if ((pending >> k) & 1u) v[k] = ld_tag2(rec0 + (size_t)(cb + k) * a.att_stride);
-      }
-#pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        if (k < ce) {  // chunk order: the same sum in every CTA
-          const float w = wv[h * nch + cb + k];
-          s0 = fmaf(w, lo_f(v[k].x), s0);
-          s1 = fmaf(w, lo_f(v[k].y), s1);
-        }
-      }
-    }
-    o[2 * p] = s0;
-    o[2 * p + 1] = s1;
-  }
-  return vote_ok(ok, pc.s_abort);
 }
 
 // Next token: argmax over the per-CTA candidates (identical in every CTA).
@@ -628,11 +639,14 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
   const unsigned per_step = (unsigned)(kPhasesPerLayer * a.L + 1);
   uint32_t g = 0;
   int token = a.start_token;
-  // x += (published vector), identically in every CTA
-  auto add_published = [&](const unsigned long long* src, unsigned tag) {
+  // x += (published vector), identically in every CTA; ss += the new x^2
+  auto add_published = [&](const unsigned long long* src, unsigned tag, float& ss) {
     const bool ok = poll_pairs(src, a.d >> 1, tag, pc, [&](int p, float v0, float v1) {
-      xs[2 * p] += v0;
-      xs[2 * p + 1] += v1;
+      const float x0 = xs[2 * p] + v0, x1 = xs[2 * p + 1] + v1;
+      xs[2 * p] = x0;
+      xs[2 * p + 1] = x1;
+      ss = fmaf(x0, x0, ss);
+      ss = fmaf(x1, x1, ss);
     });
     return vote_ok(ok, s_abort);
   };
@@ -665,14 +679,23 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
       for (int k = 0; k < 4; ++k) {
         if (k == 0 || k == 2) {
           // x += (the previous phase's published output), then x_b = RMSNorm(x, g)
+          const float* gain = reinterpret_cast<const float*>(lw + (k == 0 ? a.o_gatt : a.o_gffn));
+          Gains gp;
+          gp.load(gain, a.d);
+          float ss = 0.f;
           if (k == 2 || l > 0) {
-            if (!add_published(k == 0 ? a.x_f : a.x_o, k == 0 ? el - 1 : el + 2)) return false;
+            if (!add_published(k == 0 ? a.x_f : a.x_o, k == 0 ? el - 1 : el + 2, ss)) return false;
+          } else {
+            ss = sum_sq(xs, a.d);
           }
-          rmsnorm_to(vec, xs, reinterpret_cast<const float*>(lw + (k == 0 ? a.o_gatt : a.o_gffn)),
-                     a.d, a.eps, red);
+          rmsnorm_finish(vec, xs, gp, gain, a.d, a.eps, ss, red);
         } else if (k == 1) {
           if (!attention_phase(a, l, pos, el, el + 1, asm_, red, pc)) return false;
-          if (!merge_attention(a, pos, el + 1, vec, asm_, pc)) return false;
+          const bool ok = poll_pairs(a.x_attn, a.d >> 1, el + 1, pc, [&](int p, float v0, float v1) {
+            vec[2 * p] = v0;
+            vec[2 * p + 1] = v1;
+          });
+          if (!vote_ok(ok, s_abort)) return false;
         } else {  // h = silu(a) * b (paper §2.1, SwiGLU); a = h13[i], b = h13[F + i]
           const bool ok = poll_pairs2(a.x_h13, a.x_h13 + a.F, a.F >> 1, el + 3, pc,
                                       [&](int p, float a0, float a1, float b0, float b1) {
@@ -692,8 +715,17 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
           return false;
       }
     }
-    if (a.L > 0 && !add_published(a.x_f, es + per_step - 2)) return false;
-    rmsnorm_to(vec, xs, a.g_final, a.d, a.eps, red);
+    {
+      Gains gp;
+      gp.load(a.g_final, a.d);
+      float ss = 0.f;
+      if (a.L > 0) {
+        if (!add_published(a.x_f, es + per_step - 2, ss)) return false;
+      } else {
+        ss = sum_sq(xs, a.d);
+      }
+      rmsnorm_finish(vec, xs, gp, a.g_final, a.d, a.eps, ss, red);
+    }
     EpiArgmax ea{a.logits, -INFINITY, 0x7fffffff};
     if (!consume_phase<false>(r, g, plan_stages(a.V, a.d, a.G, c), vec, 1, a.d, seg, ea, a.err,
                        a.err_host, s_abort))
