@@ -34,6 +34,7 @@ namespace tvl {
 constexpr int kAttMinChunk = 32;    // positions per attention work item, at least
 constexpr int kAttMaxChunk = 1024;  // and at most
 constexpr int kPhasesPerLayer = 5;  // exchanges per layer: qkv, att, o, h13, f
+constexpr uint32_t kRefillDelayNs = 1000;  // producer pause before refilling freed stages
 
 struct DecodeArgs {
   // weights (inside the arena)
@@ -592,6 +593,7 @@ __device__ inline bool reduce_candidates(const DecodeArgs& a, int parity, unsign
 // layer's [Wq|Wk|Wv], Wo, [W1|W3], W2, then the classifier; this CTA's rows.
 struct DecodeSched {
   const DecodeArgs* a;
+  uint32_t refill_delay_ns = kRefillDelayNs;
   int s = 0, l = 0, k = 0;
   __device__ bool next(const float*& W, StagePlan& p) {
     if (s >= a->n_steps) return false;

@@ -41,6 +41,7 @@ struct EpiPart {
 // The single phase of a standalone GEMV.
 struct GemvSched {
   const float* W;
+  uint32_t refill_delay_ns;
   StagePlan p;
   bool given;
   __device__ bool next(const float*& w, StagePlan& plan) {
@@ -75,7 +76,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   uint32_t g = 0;
   if (threadIdx.x >= kConsumerThreads) {
     if (threadIdx.x == kConsumerThreads) {
-      GemvSched sched{a.W, p, false};
+      GemvSched sched{a.W, 0u, p, false};
       run_producer(r, sched, nullptr, nullptr, s_abort);
     }
     return;

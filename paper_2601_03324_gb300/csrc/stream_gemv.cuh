@@ -156,11 +156,19 @@ __device__ inline void run_producer(const Ring& r, Sched& sched, int* err, int* 
       if (g >= (uint32_t)r.nst) {
         bool to = false;
         const uint32_t par = ((g / (uint32_t)r.nst) - 1u) & 1u;
-        if (!wait_bounded(&r.empty[slot], par, err, s_abort, true, &to)) {
+        const bool was_free = mbar_try_wait(&r.empty[slot], par);
+        if (!was_free && !wait_bounded(&r.empty[slot], par, err, s_abort, true, &to)) {
           if (to) raise_error(err, err_host, kErrTimeout);
           *s_abort = 1;
           ok = false;
           break;
+        }
+        // Slots come back in bursts, at the end of a phase, just when the
+        // consumers start polling for that phase's exchange; refilling them
+        // at once would put a burst of HBM misses in front of those polls.
+        if (!was_free && sched.refill_delay_ns) {
+          const uint64_t t0 = globaltimer_ns();
+          while (globaltimer_ns() - t0 < sched.refill_delay_ns) {}
         }
       }
       const StageDesc s = stage_desc(p, j);
