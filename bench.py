@@ -47,7 +47,7 @@ def parse():
     ap.add_argument("--steps", type=int, default=4096)
     ap.add_argument("--warmup", type=int, default=256)
     ap.add_argument("--impl", default="tvl", choices=["tvl", "reference"])
-    ap.add_argument("--workload", default="110m", choices=["110m", "tiny", "7b"])
+    ap.add_argument("--workload", default="110m", choices=["110m", "110m-long", "tiny", "7b"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
@@ -246,10 +246,15 @@ def run_reference(args, cfg, rank, world):
 def workload_config(name, cfg):
     desc = {"110m": "110M Llama-2-shape FP32 decoder (d768 L12 H12 F2048 V32000, tied), "
                     "batch 1, greedy 256-step sequences from token 1",
-            "tiny": "tiny Llama-2-shape FP32 decoder (d288 L6 H6 F768 V32000), batch 1",
-            "7b": "7B Llama-2-shape FP32 decoder (d4096 L32 H32 F11008 V32000), batch 1, "
-                  "greedy 16-step sequences"}[name]
-    return {"workload": desc, "seq_steps": min(SEQ, cfg["max_seq"]), "batch": 1,
+            "110m-long": "110M Llama-2-shape FP32 decoder (d768 L12 H12 F2048 V32000, tied), "
+                         "batch 1, KV cache filled by 896 prompt tokens (uniform in [3, 31999], "
+                         "seed 3), greedy 128-step sequences at positions 896..1023",
+            "tiny": "tiny Llama-2-shape FP32 decoder (d288 L6 H6 F768 V32000, untied), batch 1, "
+                    "greedy 64-step sequences from token 1",
+            "7b": "7B Llama-2-shape FP32 decoder (d4096 L32 H32 F11008 V32000, untied), batch 1, "
+                  "greedy 16-step sequences from token 1"}[name]
+    seq = 128 if name == "110m-long" else min(cfg["steps"], cfg["max_seq"])
+    return {"workload": desc, "seq_steps": seq, "batch": 1,
             "weights_seed": cfg["seed"], "parallelism": "replicas",
             "l2": "inputs larger than L2: every step streams all weights (> L2 size)"}
 
@@ -298,7 +303,7 @@ def main():
     args = parse()
     rank, local_rank, world = dist_env()
     from paper_2601_03324_gb300 import synth
-    cfg = synth.model_config(args.workload)
+    cfg = synth.model_config("110m" if args.workload == "110m-long" else args.workload)
     if args.impl == "reference":
         return run_reference(args, cfg, rank, world)
     import torch
@@ -314,7 +319,17 @@ def main():
     stream = torch.cuda.Stream()
     model = tvl.Model(cfg, blob, stream=stream.cuda_stream)
     info = model.info()
-    seq = min(SEQ, cfg["max_seq"])
+    seq = min(cfg["steps"], cfg["max_seq"])  # the workload's greedy sequence length
+    tok0, pos0 = 1, 0
+    if args.workload == "110m-long":
+        # fill the KV cache with the 896-token prompt, one decode step per token;
+        # every timed sequence then decodes positions 896..1023 greedily
+        prompt = synth.long_context_tokens()
+        host = np.empty(cfg["vocab_size"], dtype=np.float32)
+        for p, t in enumerate(prompt):
+            model.forward(int(t), p, host if p == len(prompt) - 1 else None)
+        tok0, pos0 = int(np.argmax(host)), len(prompt)
+        seq = cfg["max_seq"] - pos0
 
     def run_steps(k, events=None):
         """k decode steps as greedy sequences of `seq` steps (one launch each)."""
@@ -325,7 +340,7 @@ def main():
             if events is not None:
                 e0 = torch.cuda.Event(enable_timing=True)
                 e0.record(stream)
-            model.decode_greedy(1, 0, n, tokens=False)
+            model.decode_greedy(tok0, pos0, n, tokens=False)
             if events is not None:
                 e1 = torch.cuda.Event(enable_timing=True)
                 e1.record(stream)
@@ -364,7 +379,7 @@ def main():
     full = [(a.elapsed_time(b), n) for (a, b, n) in ev]
     launch_ms = statistics.mean(t for t, n in full)
     n_typ = full[0][1]
-    bytes_launch = sum(step_bytes(cfg, info.streamed_bytes, p) for p in range(n_typ))
+    bytes_launch = sum(step_bytes(cfg, info.streamed_bytes, pos0 + p) for p in range(n_typ))
     peak, peak_src = measured_peaks()
     achieved = bytes_launch / (statistics.mean(t for t, n in full if n == n_typ) * 1e-3) / 1e9
     traffic = committed_traffic(args.workload, bytes_launch)
@@ -377,18 +392,18 @@ def main():
         import torch as _t
         host_logits = _t.empty(cfg["vocab_size"], dtype=_t.float32, pin_memory=True).numpy()
         k_e2e = min(args.steps, 2048)
-        tok = 1
-        for p in range(8):
+        tok = tok0
+        for p in range(pos0, pos0 + 8):
             model.forward(tok, p, host_logits)
             tok = int(np.argmax(host_logits))
         t0 = time.perf_counter()
-        tok, pos = 1, 0
+        tok, pos = tok0, pos0
         for s in range(k_e2e):
             model.forward(tok, pos, host_logits)
             tok = int(np.argmax(host_logits))
             pos += 1
-            if pos == seq:
-                tok, pos = 1, 0
+            if pos == pos0 + seq:
+                tok, pos = tok0, pos0
         e2e_s = time.perf_counter() - t0
         e2e = {"value": world * k_e2e / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": 4,
                "d2h_bytes_per_step": 4 * cfg["vocab_size"],
@@ -396,7 +411,7 @@ def main():
                        "memory, argmax on the host"}
 
     cpu = None
-    if rank == 0 and not args.no_cpu_baseline and args.workload != "7b":
+    if rank == 0 and not args.no_cpu_baseline and args.workload in ("110m", "tiny"):
         rate, n, el = cpu_oracle_rate(cfg, blob, args.cpu_seconds)
         cpu = {"value": rate, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                "sample": f"first {n} greedy steps of the workload from token 1 "
