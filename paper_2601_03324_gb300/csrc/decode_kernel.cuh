@@ -382,6 +382,29 @@ struct EpiArgmax {
 
 // ---- attention -------------------------------------------------------------------
 
+// Ask L2 for the K/V rows (positions before pos) that this CTA's attention
+// items of layer l will read: the cache lines are usually no longer in L2
+// (the weight stream has gone through it since), and the request is issued a
+// phase ahead so that the items' own loads find them there.
+__device__ inline void att_prefetch_l2(const DecodeArgs& a, int l, int pos) {
+  int nch, clen;
+  att_split(pos, a.H, a.G, &nch, &clen);
+  const int group = a.H / a.Hkv, hd = a.hd;
+  const int lpr = (hd * 4 + 127) / 128;  // 128-byte lines per row
+  const size_t lay = (size_t)l * a.S * a.kvd;
+  for (int it = blockIdx.x; it < a.H * nch; it += a.G) {
+    const int h = it / nch, c = it - h * nch, kvh = h / group;
+    const int t0 = c * clen, te = (t0 + clen < pos) ? t0 + clen : pos;
+    const int per = (te - t0) * lpr;
+    for (int i = threadIdx.x; i < 2 * per; i += kConsumerThreads) {
+      const int which = i >= per, rem = i - which * per;
+      const int t = t0 + rem / lpr, ln = rem - (rem / lpr) * lpr;
+      const float* q = (which ? a.vc : a.kc) + lay + (size_t)t * a.kvd + kvh * hd + ln * 32;
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(q));
+    }
+  }
+}
+
 // Attention partials of this CTA's items for layer l at position pos. Item
 // (h, c): query head h over the positions of chunk c; publishes the chunk's
 // max score m, sum of exp(s - m), and sum of exp(s - m) * v.
@@ -679,6 +702,7 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
       const unsigned el = es + (unsigned)(kPhasesPerLayer * l);
 #pragma unroll 1
       for (int k = 0; k < 4; ++k) {
+        if (k == 0) att_prefetch_l2(a, l, pos);
         if (k == 0 || k == 2) {
           // x += (the previous phase's published output), then x_b = RMSNorm(x, g)
           const float* gain = reinterpret_cast<const float*>(lw + (k == 0 ? a.o_gatt : a.o_gffn));
