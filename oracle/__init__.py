@@ -68,6 +68,13 @@ def lib():
         L.orc_model_new.restype = P
         L.orc_model_new.argtypes = [ctypes.POINTER(Config), P, ctypes.c_size_t, ctypes.c_int,
                                     ctypes.POINTER(ctypes.c_int)]
+        L.orc_model_new_fmt.restype = P
+        L.orc_model_new_fmt.argtypes = [ctypes.POINTER(Config), P, ctypes.c_size_t, ctypes.c_int,
+                                        ctypes.c_int, ctypes.POINTER(ctypes.c_int)]
+        L.orc_quantize_rows_q8.restype = None
+        L.orc_quantize_rows_q8.argtypes = [P, i64, i64, P, P]
+        L.orc_gemv_q8_f64.restype = None
+        L.orc_gemv_q8_f64.argtypes = [P, P, P, P, i64, i64]
         L.orc_forward.restype = ctypes.c_int
         L.orc_forward.argtypes = [P, i32, i32, P]
         L.orc_model_tied.restype = ctypes.c_int
@@ -108,6 +115,27 @@ def gemv(W: np.ndarray, x: np.ndarray, acc_bits: int = 64) -> np.ndarray:
         x = np.ascontiguousarray(x, dtype=np.float32)
         y = np.empty(M, dtype=np.float32)
         lib().orc_gemv_f32(_ptr(W), _ptr(x), _ptr(y), M, K)
+    return y
+
+
+def quantize_rows_q8(W: np.ndarray):
+    """8-bit codes and row scales of W float32 [M, K] (see orc_quantize_rows_q8)."""
+    W = np.ascontiguousarray(W, dtype=np.float32)
+    M, K = W.shape
+    q = np.empty((M, K), dtype=np.int8)
+    s = np.empty(M, dtype=np.float32)
+    lib().orc_quantize_rows_q8(_ptr(W), M, K, _ptr(q), _ptr(s))
+    return q, s
+
+
+def gemv_q8(q: np.ndarray, s: np.ndarray, x: np.ndarray) -> np.ndarray:
+    """y = (s_i q_ij) x in double."""
+    q = np.ascontiguousarray(q, dtype=np.int8)
+    s = np.ascontiguousarray(s, dtype=np.float32)
+    x = np.ascontiguousarray(x, dtype=np.float64)
+    M, K = q.shape
+    y = np.empty(M, dtype=np.float64)
+    lib().orc_gemv_q8_f64(_ptr(q), _ptr(s), _ptr(x), _ptr(y), M, K)
     return y
 
 
@@ -159,13 +187,15 @@ def tensor_offset(cfg: dict, tied: bool, which: int, layer: int = 0) -> int:
 class Model:
     """One decode session of the oracle over a borrowed blob (numpy array kept alive)."""
 
-    def __init__(self, cfg: dict, blob: np.ndarray, acc_bits: int = 64):
+    def __init__(self, cfg: dict, blob: np.ndarray, acc_bits: int = 64, weight_bits: int = 0):
+        """weight_bits 8: every weight matrix as 8-bit codes with row scales."""
         self._blob = blob  # keep alive
         self.cfg = dict(cfg)
         c = make_config(cfg)
         err = ctypes.c_int(0)
-        self._h = lib().orc_model_new(ctypes.byref(c), ctypes.c_void_p(blob.ctypes.data),
-                                      blob.nbytes, acc_bits, ctypes.byref(err))
+        self._h = lib().orc_model_new_fmt(ctypes.byref(c), ctypes.c_void_p(blob.ctypes.data),
+                                          blob.nbytes, acc_bits, int(weight_bits),
+                                          ctypes.byref(err))
         if not self._h:
             raise ValueError(f"orc_model_new failed with code {err.value}")
         self.vocab = int(cfg["vocab_size"])

@@ -16,6 +16,9 @@
 //   * Attention over a KV cache, one new token per step— §1 (decode is GEMV
 //     bound, every weight read once per token) and §2.1 (Llama 2 decoder).
 //   * Classifier tied to the token embedding when the file is short — §5.1.
+//   * Weight-only 8-bit codes with one scale per output row: a reading of
+//     the quantization the paper leaves to future work (§ Future Work:
+//     Quantization, which names 4-bit weights unpacked on the fly).
 // Where the paper is silent, the readings taken are the standard Llama-2
 // ones and are listed where they are used.
 //
@@ -24,6 +27,7 @@
 // reordering of any sum: every loop runs in index order.
 #include "orc.h"
 
+#include <cfenv>
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
@@ -96,6 +100,42 @@ void gemv(const float* W, const Acc* x, Acc* y, int64_t M, int64_t K) {
     Acc s = 0;
     for (int64_t j = 0; j < K; ++j) s += (Acc)w[j] * x[j];
     y[i] = s;
+  }
+}
+
+// Weight-only 8-bit codes, one float32 scale per output row. Every decision
+// is taken in float32, so that any implementation of the same definition
+// finds the same codes: a_r = max_j |W_rj|; s_r = a_r / 127; q_rj = the
+// integer nearest to W_rj / s_r (ties to even), which lies in [-127, 127];
+// an all-zero row has s_r = 0 and codes 0. The weight a code stands for is
+// s_r * q_rj.
+void quantize_rows(const float* W, int64_t M, int64_t K, int8_t* q, float* s) {
+  for (int64_t i = 0; i < M; ++i) {
+    const float* w = W + i * K;
+    float a = 0.0f;
+    for (int64_t j = 0; j < K; ++j) a = std::fmax(a, std::fabs(w[j]));
+    const float sc = a / 127.0f;
+    s[i] = sc;
+    for (int64_t j = 0; j < K; ++j) {
+      float c = 0.0f;
+      if (sc != 0.0f) {
+        c = std::nearbyint(w[j] / sc);  // default rounding: nearest, ties to even
+        if (c > 127.0f) c = 127.0f;
+        if (c < -127.0f) c = -127.0f;
+      }
+      q[i * K + j] = (int8_t)c;
+    }
+  }
+}
+
+// y[i] = sum_j (s_i q_ij) x[j]: the GEMV of the weights the codes stand for.
+template <class Acc>
+void gemv_q8(const int8_t* q, const float* s, const Acc* x, Acc* y, int64_t M, int64_t K) {
+  for (int64_t i = 0; i < M; ++i) {
+    const int8_t* c = q + i * K;
+    Acc acc = 0;
+    for (int64_t j = 0; j < K; ++j) acc += ((Acc)s[i] * (Acc)c[j]) * x[j];
+    y[i] = acc;
   }
 }
 
@@ -173,11 +213,25 @@ struct ModelBase {
   bool tied = false;
 };
 
+// One weight matrix as 8-bit codes and row scales.
+struct QMat {
+  std::vector<int8_t> q;
+  std::vector<float> s;
+  void make(const float* W, int64_t M, int64_t K) {
+    q.resize((size_t)(M * K));
+    s.resize((size_t)M);
+    quantize_rows(W, M, K, q.data(), s.data());
+  }
+};
+
 template <class Acc>
 struct Model : ModelBase {
   orc_config c;
   const char* blob;
   Layout L;
+  bool q8 = false;  // weight matrices as 8-bit codes (gains stay float32)
+  std::vector<QMat> qWq, qWk, qWv, qWo, qW1, qW3, qW2;
+  QMat qE, qWcls;
   int64_t d, F, V, H, Hkv, hd, kvd, S;
   std::vector<Acc> x, xb, q, k, v, o, a, b, hb, y, att, logit;
   Acc* kcache = nullptr;  // [L][S][kvd]
@@ -202,19 +256,49 @@ struct Model : ModelBase {
     return kcache && vcache;
   }
 
+  // Codes of every weight matrix (the embedding table too; it is also the
+  // classifier when tied).
+  void quantize_all() {
+    q8 = true;
+    const int nl = c.n_layers;
+    qWq.resize(nl); qWk.resize(nl); qWv.resize(nl); qWo.resize(nl);
+    qW1.resize(nl); qW3.resize(nl); qW2.resize(nl);
+    for (int l = 0; l < nl; ++l) {
+      qWq[l].make(T(L.Wq[l]), d, d);
+      qWk[l].make(T(L.Wk[l]), kvd, d);
+      qWv[l].make(T(L.Wv[l]), kvd, d);
+      qWo[l].make(T(L.Wo[l]), d, d);
+      qW1[l].make(T(L.W1[l]), F, d);
+      qW3[l].make(T(L.W3[l]), F, d);
+      qW2[l].make(T(L.W2[l]), d, F);
+    }
+    qE.make(T(L.E), V, d);
+    if (!tied) qWcls.make(T(L.Wcls), V, d);
+  }
+  void mv(const std::vector<QMat>& qm, const std::vector<int64_t>& off, int l, const Acc* xin,
+          Acc* yout, int64_t M, int64_t K) {
+    if (q8) gemv_q8(qm[l].q.data(), qm[l].s.data(), xin, yout, M, K);
+    else gemv(T(off[l]), xin, yout, M, K);
+  }
+
   int forward(int32_t token, int32_t pos, double* logits) override {
     if (token < 0 || token >= V || pos < 0 || pos >= S) return 6;
     const Acc eps = (Acc)c.norm_eps;
     // token embedding row (§4.1: weights are pointers at offsets in the blob)
-    const float* e = T(L.E) + (int64_t)token * d;
-    for (int64_t j = 0; j < d; ++j) x[j] = (Acc)e[j];
+    if (q8) {
+      const int8_t* qe = qE.q.data() + (size_t)token * d;
+      for (int64_t j = 0; j < d; ++j) x[j] = (Acc)qE.s[token] * (Acc)qe[j];
+    } else {
+      const float* e = T(L.E) + (int64_t)token * d;
+      for (int64_t j = 0; j < d; ++j) x[j] = (Acc)e[j];
+    }
 
     for (int l = 0; l < c.n_layers; ++l) {
       // attention block
       rmsnorm(x.data(), T(L.g_att[l]), xb.data(), d, eps);
-      gemv(T(L.Wq[l]), xb.data(), q.data(), d, d);
-      gemv(T(L.Wk[l]), xb.data(), k.data(), kvd, d);
-      gemv(T(L.Wv[l]), xb.data(), v.data(), kvd, d);
+      mv(qWq, L.Wq, l, xb.data(), q.data(), d, d);
+      mv(qWk, L.Wk, l, xb.data(), k.data(), kvd, d);
+      mv(qWv, L.Wv, l, xb.data(), v.data(), kvd, d);
       rope(q.data(), d, hd, pos, c.rope_theta);
       rope(k.data(), kvd, hd, pos, c.rope_theta);
       Acc* Kc = kcache + (size_t)l * S * kvd;
@@ -230,20 +314,25 @@ struct Model : ModelBase {
         attention_head(q.data() + h * hd, Kc + kvh * hd, Vc + kvh * hd, (int64_t)pos + 1, hd,
                        kvd, o.data() + h * hd, att.data());
       }
-      gemv(T(L.Wo[l]), o.data(), y.data(), d, d);
+      mv(qWo, L.Wo, l, o.data(), y.data(), d, d);
       for (int64_t j = 0; j < d; ++j) x[j] = x[j] + y[j];
 
       // feed-forward block: W2 (silu(W1 xb) * (W3 xb))
       rmsnorm(x.data(), T(L.g_ffn[l]), xb.data(), d, eps);
-      gemv(T(L.W1[l]), xb.data(), a.data(), F, d);
-      gemv(T(L.W3[l]), xb.data(), b.data(), F, d);
+      mv(qW1, L.W1, l, xb.data(), a.data(), F, d);
+      mv(qW3, L.W3, l, xb.data(), b.data(), F, d);
       for (int64_t i = 0; i < F; ++i) hb[i] = silu(a[i]) * b[i];
-      gemv(T(L.W2[l]), hb.data(), y.data(), d, F);
+      mv(qW2, L.W2, l, hb.data(), y.data(), d, F);
       for (int64_t j = 0; j < d; ++j) x[j] = x[j] + y[j];
     }
     rmsnorm(x.data(), T(L.g_final), xb.data(), d, eps);
     // classifier; §5.1: W_cls is the embedding table when tied
-    gemv(T(tied ? L.E : L.Wcls), xb.data(), logit.data(), V, d);
+    if (q8) {
+      const QMat& qc = tied ? qE : qWcls;
+      gemv_q8(qc.q.data(), qc.s.data(), xb.data(), logit.data(), V, d);
+    } else {
+      gemv(T(tied ? L.E : L.Wcls), xb.data(), logit.data(), V, d);
+    }
     for (int64_t i = 0; i < V; ++i) logits[i] = (double)logit[i];
     return 0;
   }
@@ -281,10 +370,16 @@ int64_t orc_tensor_offset(const orc_config* cfg, int tied, int which, int layer)
 
 void* orc_model_new(const orc_config* cfg, const void* blob, size_t blob_bytes, int acc_bits,
                     int* err) {
+  return orc_model_new_fmt(cfg, blob, blob_bytes, acc_bits, 0, err);
+}
+
+void* orc_model_new_fmt(const orc_config* cfg, const void* blob, size_t blob_bytes, int acc_bits,
+                        int weight_bits, int* err) {
   int dummy;
   if (!err) err = &dummy;
   *err = 0;
-  if (!config_ok(cfg) || !blob || (acc_bits != 32 && acc_bits != 64)) {
+  if (!config_ok(cfg) || !blob || (acc_bits != 32 && acc_bits != 64) ||
+      (weight_bits != 0 && weight_bits != 8)) {
     *err = 1;
     return nullptr;
   }
@@ -314,6 +409,10 @@ void* orc_model_new(const orc_config* cfg, const void* blob, size_t blob_bytes, 
   }
   if (!m) { *err = 4; return nullptr; }
   m->tied = tied;
+  if (weight_bits == 8) {
+    if (acc_bits == 64) static_cast<Model<double>*>(m)->quantize_all();
+    else static_cast<Model<float>*>(m)->quantize_all();
+  }
   return m;
 }
 
@@ -325,6 +424,15 @@ int orc_forward(void* model, int32_t token, int32_t pos, double* logits) {
 int orc_model_tied(const void* model) { return model ? (int)((const ModelBase*)model)->tied : -1; }
 
 void orc_model_free(void* model) { delete (ModelBase*)model; }
+
+void orc_quantize_rows_q8(const float* W, int64_t M, int64_t K, int8_t* q, float* s) {
+  quantize_rows(W, M, K, q, s);
+}
+
+void orc_gemv_q8_f64(const int8_t* q, const float* s, const double* x, double* y, int64_t M,
+                     int64_t K) {
+  gemv_q8<double>(q, s, x, y, M, K);
+}
 
 void orc_gemv_f64(const float* W, const double* x, double* y, int64_t M, int64_t K) {
   gemv<double>(W, x, y, M, K);

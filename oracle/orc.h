@@ -42,6 +42,11 @@ int64_t orc_tensor_offset(const orc_config* cfg, int tied, int which, int layer)
  * Returns NULL and sets *err (1 invalid config, 2 size mismatch, 4 no memory). */
 void* orc_model_new(const orc_config* cfg, const void* blob, size_t blob_bytes,
                     int acc_bits, int* err);
+/* Same, with every weight matrix replaced by 8-bit codes and row scales
+ * (weight_bits 8; 0 keeps float32), quantized at construction as
+ * orc_quantize_rows_q8 defines. */
+void* orc_model_new_fmt(const orc_config* cfg, const void* blob, size_t blob_bytes,
+                        int acc_bits, int weight_bits, int* err);
 /* One decode step (token at position pos); writes vocab_size logits.
  * Returns 0, or 6 when token/pos is out of range. */
 int orc_forward(void* model, int32_t token, int32_t pos, double* logits);
@@ -49,6 +54,13 @@ int orc_model_tied(const void* model);
 void orc_model_free(void* model);
 
 /* Primitives, exposed so that tests can pin each one on its own. */
+/* Weight-only 8-bit codes of W [M x K]: s[i] = max_j |W[i][j]| / 127 and
+ * q[i][j] = nearest integer (ties to even) to W[i][j] / s[i], all in float32
+ * (0 codes and scale for an all-zero row). */
+void orc_quantize_rows_q8(const float* W, int64_t M, int64_t K, int8_t* q, float* s);
+/* y[i] = sum_j (s[i] * q[i][j]) * x[j] in double. */
+void orc_gemv_q8_f64(const int8_t* q, const float* s, const double* x, double* y, int64_t M,
+                     int64_t K);
 void orc_gemv_f64(const float* W, const double* x, double* y, int64_t M, int64_t K);
 void orc_gemv_f32(const float* W, const float* x, float* y, int64_t M, int64_t K);
 void orc_rmsnorm_f64(const double* x, const float* g, double* out, int64_t n, double eps);

@@ -327,3 +327,86 @@ def test_float_and_double_oracles_agree_within_decode_tolerances():
         top2 = np.sort(ref)[-2:]
         if top2[1] - top2[0] > 1e-2:
             assert int(np.argmax(got)) == int(np.argmax(ref))
+
+
+# ---- weight-only 8-bit codes (the paper's quantization future work, read as
+# per-row symmetric 8-bit codes: s = max|w| / 127, q = nearest(w / s), ties to even) ----
+
+def test_q8_integer_rows_with_max_127_keep_their_values_and_round_ties_to_even():
+    W = np.array([[127, 0.5, 1.5, 2.5, -0.5, -1.5, 3.5, -2.5, -127, 64]], np.float32)
+    q, s = oracle.quantize_rows_q8(W)
+    assert s[0] == np.float32(1.0)
+    assert q.tolist() == [[127, 0, 2, 2, 0, -2, 4, -2, -127, 64]]
+
+
+def test_q8_zero_row_sign_symmetry_and_power_of_two_scaling():
+    W = RNG.standard_normal((9, 33)).astype(np.float32)
+    W[4] = 0.0
+    q, s = oracle.quantize_rows_q8(W)
+    assert s[4] == 0.0 and not q[4].any()
+    qn, sn = oracle.quantize_rows_q8(-W)
+    assert np.array_equal(qn, -q) and np.array_equal(sn, s)
+    q8, s8 = oracle.quantize_rows_q8(W * np.float32(8.0))  # exact in float32
+    assert np.array_equal(q8, q) and np.array_equal(s8, s * np.float32(8.0))
+
+
+def test_q8_codes_reach_127_at_the_row_maximum_and_stay_within_half_a_step():
+    W = (RNG.standard_normal((40, 200)) * 0.02).astype(np.float32)
+    q, s = oracle.quantize_rows_q8(W)
+    for i in range(40):
+        j = int(np.argmax(np.abs(W[i])))
+        assert abs(int(q[i, j])) == 127
+        assert np.abs(q[i]).max() == 127
+        err = np.abs(W[i].astype(np.float64) - float(s[i]) * q[i].astype(np.float64))
+        assert err.max() <= 0.5 * float(s[i]) * (1 + 1e-6)  # nearest code, float32 division
+    assert float(s[0]) == float(np.float32(np.abs(W[0]).max()) / np.float32(127.0))
+
+
+def test_q8_gemv_is_the_gemv_of_the_weights_the_codes_stand_for():
+    q = RNG.integers(-127, 128, size=(7, 13)).astype(np.int8)
+    s = (RNG.random(7) * 0.01).astype(np.float32)
+    x = RNG.standard_normal(13)
+    y = oracle.gemv_q8(q, s, x)
+    for i in range(7):
+        exact = sum(Fraction(float(s[i])) * int(q[i, j]) * Fraction(float(x[j])) for j in range(13))
+        bound = 13 * 2.0 ** -51 * sum(abs(float(s[i]) * int(q[i, j]) * x[j]) for j in range(13))
+        assert abs(Fraction(y[i]) - exact) <= Fraction(bound)
+    eye = np.eye(13, dtype=np.int8) * 127
+    assert np.allclose(oracle.gemv_q8(eye, np.full(13, 1 / 127, np.float32), x),
+                       x * 127 * float(np.float32(1 / 127)), rtol=0, atol=1e-15)
+
+
+def _representable_blob(cfg, seed):
+    """A blob whose every weight matrix row is k * 2^-12 with integer |k| <= 127
+    and some |k| == 127: its 8-bit codes and scales are exact."""
+    blob = synth.make_blob(cfg, seed=seed)
+    names = ["Wq", "Wk", "Wv", "Wo", "W1", "W3", "W2"]
+    mats = [("E", -1)] + [(n, l) for l in range(cfg["n_layers"]) for n in names]
+    if not cfg["shared_classifier"]:
+        mats.append(("Wcls", -1))
+    for (n, l) in mats:
+        T = synth.tensor(blob, cfg, n, l)
+        k = np.clip(np.rint(T * 4096.0), -127, 127)
+        k[:, 0] = np.where(k[:, 0] < 0, -127, 127)
+        T[...] = (k / 4096.0).astype(np.float32)
+    return blob
+
+
+@pytest.mark.parametrize("tied", [1, 0])
+def test_q8_model_equals_float_model_on_exactly_representable_weights(tied):
+    cfg = dict(synth.model_config("tiny"), n_layers=2, vocab_size=500, max_seq=8,
+               shared_classifier=tied)
+    blob = _representable_blob(cfg, 5)
+    mf = oracle.Model(cfg, blob)
+    mq = oracle.Model(cfg, blob, weight_bits=8)
+    for pos, tok in enumerate([3, 17, 499, 0, 250]):
+        assert np.array_equal(mq.forward(tok, pos), mf.forward(tok, pos))
+
+
+def test_q8_model_differs_from_float_model_by_quantization_only():
+    cfg = dict(synth.model_config("tiny"), n_layers=2, vocab_size=500, max_seq=8)
+    blob = synth.make_blob(cfg, seed=6)
+    lf = oracle.Model(cfg, blob).forward(1, 0)
+    lq = oracle.Model(cfg, blob, weight_bits=8).forward(1, 0)
+    rel = np.abs(lq - lf).max() / np.abs(lf).max()
+    assert 1e-5 < rel < 5e-2  # the codes change the result, by about the code step
