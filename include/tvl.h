@@ -119,6 +119,30 @@ tvl_status tvl_decode_greedy(tvl_model* m, int32_t start_token, int32_t start_po
 tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t d_out, int32_t d_in,
                     void* stream);
 
+/* Weight-only 8-bit rows. The paper leaves quantization to future work
+ * (§ Future Work: Quantization: narrow weights unpacked on the fly, for less
+ * memory traffic per token); this is one reading of it. A matrix W [rows x
+ * cols] becomes packed rows of 16 + cols bytes each: the float32 scale
+ * s = max_j |W[r][j]| / 127 (bytes 0-3), twelve zero bytes, then the codes
+ * q[r][j] = the integer nearest to W[r][j] / s (ties to even, in [-127, 127];
+ * an all-zero row has s = 0 and codes 0), every step in float32. The code
+ * stands for the weight s * q. cols must be a positive multiple of 16.
+ * tvl_q8_bytes: bytes of the packed rows (0 if rows < 1 or cols is invalid). */
+size_t tvl_q8_bytes(int32_t rows, int32_t cols);
+
+/* Quantize W (device, float32, row-major, 16-byte aligned) into Wq8 (device,
+ * tvl_q8_bytes(rows, cols) bytes, 16-byte aligned), on `stream`, without
+ * waiting. Errors: TVL_E_INVAL (null pointer, bad size), TVL_E_ALIGN. */
+tvl_status tvl_quantize_q8(const float* W, void* Wq8, int32_t rows, int32_t cols, void* stream);
+
+/* y = W' x for the weights W' the packed rows stand for (y[r] = s_r * sum_j
+ * q[r][j] x[j]); Wq8 and x device pointers, 16-byte aligned; d_in a multiple
+ * of 16 and at most 16368 (a packed row fits one 16 KB stage), else
+ * TVL_E_INVAL / TVL_E_UNSUPPORTED. Queued on `stream`, does not wait,
+ * allocates nothing. */
+tvl_status tvl_gemv_q8(const void* Wq8, const float* x, float* y, int32_t d_out, int32_t d_in,
+                       void* stream);
+
 /* tvl_gemv without any allocation. The paper has no counterpart: this entry
  * exists for callers that cannot allocate device memory at call time — a host
  * thread that must not stall other streams (cudaMalloc and cudaFree may

@@ -288,6 +288,37 @@ __device__ __forceinline__ float row_partial_xr(const float4* w4, const float4 (
   return ((c0.x + c0.y) + (c0.z + c0.w)) + ((c1.x + c1.y) + (c1.z + c1.w));
 }
 
+// 8-bit weight rows (weight-only codes, one scale per row). A packed row is
+// 16 + K bytes: the float32 scale, 12 zero bytes, then K int8 codes; in a
+// stage a row is Kw = 4 + K/4 words. Code word e holds codes 4e..4e+3 and
+// meets x float4 e.
+__device__ __forceinline__ void fma_codes(float4& acc, int w, const float4& x) {
+  acc.x = fmaf((float)(int)(signed char)(w & 0xff), x.x, acc.x);
+  acc.y = fmaf((float)(int)(signed char)((w >> 8) & 0xff), x.y, acc.y);
+  acc.z = fmaf((float)(int)(signed char)((w >> 16) & 0xff), x.z, acc.z);
+  acc.w = fmaf((float)(w >> 24), x.w, acc.w);
+}
+
+// Lane partials of sum_j q_j x_j for two 8-bit rows sharing x (nw code words).
+__device__ __forceinline__ float2 row2_partial_q8(const int* c0, const int* c1, const float4* x4,
+                                                  int nw, int lane) {
+  float4 a = make_float4(0.f, 0.f, 0.f, 0.f), b = a;
+#pragma unroll 2
+  for (int e = lane; e < nw; e += 32) {
+    const float4 x = x4[e];
+    fma_codes(a, c0[e], x);
+    fma_codes(b, c1[e], x);
+  }
+  return make_float2((a.x + a.y) + (a.z + a.w), (b.x + b.y) + (b.z + b.w));
+}
+
+__device__ __forceinline__ float row_partial_q8(const int* c0, const float4* x4, int nw, int lane) {
+  float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 2
+  for (int e = lane; e < nw; e += 32) fma_codes(a, c0[e], x4[e]);
+  return (a.x + a.y) + (a.z + a.w);
+}
+
 // Warp-level bounded wait for stage gs in `slot` (all lanes poll, lane 0
 // applies the limit): first until the producer has queued that stage into the
 // slot, then until its bytes have landed. Returns the same answer in every
@@ -350,14 +381,14 @@ __device__ inline bool warp_wait_full(const Ring& r, int slot, uint32_t gs, int*
 // that adds the row's segment partials at the end of the phase. seg is
 // shared scratch for those partials. Ends with a barrier of the consumer
 // warps; returns false on abort, identically in every consumer thread.
-template <bool kXReg = true, class Epi>
+template <bool kXReg = true, bool kQ8 = false, class Epi>
 __device__ inline bool consume_phase(const Ring& r, uint32_t& g, const StagePlan& p,
                                      const float* xs, int S, int Kc, float* seg, Epi& epi,
                                      int* err, int* err_host, volatile int* s_abort) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // Rows of at most 1024 floats (whole rows in a stage, one K-chunk): each lane
   // keeps its x slice in registers for the whole phase.
-  const bool xreg = kXReg && (p.spr == 1) && (p.K <= 1024) && (S == 1);
+  const bool xreg = kXReg && !kQ8 && (p.spr == 1) && (p.K <= 1024) && (S == 1);
   float4 xr[8];
   if (xreg) {
     const float4* x4 = reinterpret_cast<const float4*>(xs);
@@ -380,6 +411,35 @@ __device__ inline bool consume_phase(const Ring& r, uint32_t& g, const StagePlan
     const StageDesc s = stage_desc(p, j);
     const int ncols = s.c1 - s.c0, n4 = ncols >> 2;
     const float* st = reinterpret_cast<const float*>(r.buf + (size_t)slot * kStageBytes);
+    if (kQ8) {  // whole 8-bit rows (ncols = Kw words): y = scale * sum q x
+      const float4* x4 = reinterpret_cast<const float4*>(xs);
+      for (int ri = 0; ri < s.nrows; ri += 2) {
+        const bool two = ri + 1 < s.nrows;
+        const float* r0 = st + (size_t)ri * ncols;
+        const float* r1 = r0 + ncols;
+        float a0, a1 = 0.f;
+        if (two) {
+          const float2 t = row2_partial_q8(reinterpret_cast<const int*>(r0 + 4),
+                                           reinterpret_cast<const int*>(r1 + 4), x4, ncols - 4, lane);
+          a0 = t.x;
+          a1 = t.y;
+        } else {
+          a0 = row_partial_q8(reinterpret_cast<const int*>(r0 + 4), x4, ncols - 4, lane);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          a0 += __shfl_xor_sync(0xffffffffu, a0, o);
+          a1 += __shfl_xor_sync(0xffffffffu, a1, o);
+        }
+        if (lane == 0) {
+          epi.store(s.row + ri, r0[0] * a0);
+          if (two) epi.store(s.row + ri + 1, r1[0] * a1);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&r.empty[slot]);  // stage free for the producer
+      continue;
+    }
     for (int ri = 0; ri < s.nrows; ri += 2) {
       const bool two = ri + 1 < s.nrows;
       const int v0 = s.row + ri, v1 = v0 + 1;

@@ -64,6 +64,12 @@ def _load():
     L.tvl_decode_greedy.argtypes = [P, i32, i32, i32, P]
     L.tvl_gemv.restype = st
     L.tvl_gemv.argtypes = [P, P, P, i32, i32, P]
+    L.tvl_q8_bytes.restype = sz
+    L.tvl_q8_bytes.argtypes = [i32, i32]
+    L.tvl_quantize_q8.restype = st
+    L.tvl_quantize_q8.argtypes = [P, P, i32, i32, P]
+    L.tvl_gemv_q8.restype = st
+    L.tvl_gemv_q8.argtypes = [P, P, P, i32, i32, P]
     L.tvl_gemv_noalloc.restype = st
     L.tvl_gemv_noalloc.argtypes = [P, P, P, i32, i32, P]
     L.tvl_sync.restype = st
@@ -86,7 +92,8 @@ def _load():
 lib = _load()
 
 EXPORTED = ["tvl_blob_bytes", "tvl_load", "tvl_load_file", "tvl_forward", "tvl_decode_greedy",
-            "tvl_gemv", "tvl_gemv_noalloc", "tvl_sync", "tvl_free", "tvl_status_string", "tvl_last_error",
+            "tvl_gemv", "tvl_gemv_noalloc", "tvl_q8_bytes", "tvl_quantize_q8", "tvl_gemv_q8",
+            "tvl_sync", "tvl_free", "tvl_status_string", "tvl_last_error",
             "tvl_get_info", "tvl_step_times", "tvl_selftest_barrier_timeout"]
 
 
@@ -136,6 +143,23 @@ def tvl_gemv_noalloc(W, x, y, d_out: int, d_in: int, stream: int = 0):
     _check(lib.tvl_gemv_noalloc(ctypes.c_void_p(_addr(W)), ctypes.c_void_p(_addr(x)),
                                 ctypes.c_void_p(_addr(y)), int(d_out), int(d_in),
                                 ctypes.c_void_p(int(stream))), "tvl_gemv_noalloc")
+
+
+def tvl_q8_bytes(rows: int, cols: int) -> int:
+    return int(lib.tvl_q8_bytes(int(rows), int(cols)))
+
+
+def tvl_quantize_q8(W, Wq8, rows: int, cols: int, stream: int = 0):
+    """Packed 8-bit rows of W (device addresses)."""
+    _check(lib.tvl_quantize_q8(ctypes.c_void_p(_addr(W)), ctypes.c_void_p(_addr(Wq8)), int(rows),
+                               int(cols), ctypes.c_void_p(int(stream))), "tvl_quantize_q8")
+
+
+def tvl_gemv_q8(Wq8, x, y, d_out: int, d_in: int, stream: int = 0):
+    """y = W' x over packed 8-bit rows (device addresses)."""
+    _check(lib.tvl_gemv_q8(ctypes.c_void_p(_addr(Wq8)), ctypes.c_void_p(_addr(x)),
+                           ctypes.c_void_p(_addr(y)), int(d_out), int(d_in),
+                           ctypes.c_void_p(int(stream))), "tvl_gemv_q8")
 
 
 def tvl_selftest_barrier_timeout(limit_ms: int) -> int:

@@ -94,3 +94,10 @@ def test_null_and_bad_arguments(tvl):
     assert L.tvl_load(None, None, 0, None, None) == tvl.E_INVAL
     assert "range" in tvl.status_string(tvl.E_RANGE)
     assert tvl.status_string(99) == "unknown status"
+
+
+def test_q8_row_bytes_on_the_host(tvl):
+    assert tvl.tvl_q8_bytes(3, 32) == 3 * 48
+    assert tvl.tvl_q8_bytes(32000, 768) == 32000 * 784
+    for rows, cols in ((0, 32), (3, 8), (3, 24), (3, 0), (-1, 16)):
+        assert tvl.tvl_q8_bytes(rows, cols) == 0
