@@ -50,6 +50,10 @@ typedef struct {
   double rope_theta;    /* RoPE base (10000) */
   double norm_eps;      /* RMSNorm epsilon, added to mean(x^2) inside the sqrt (1e-5, §11.2) */
   int32_t shared_classifier; /* 1 tied (Wcls is E), 0 untied, -1 infer from blob size (§5.1) */
+  int32_t weight_bits;  /* 0: float32 weights as in the blob; 8: tvl_load turns every weight
+                           matrix (and the embedding table) into 8-bit rows, as
+                           tvl_quantize_q8 defines, and decodes with them; dim and
+                           hidden_dim must then be multiples of 16 */
 } tvl_config;
 
 typedef struct tvl_model tvl_model; /* opaque: device arena, stream, kernel plan */
@@ -119,7 +123,8 @@ tvl_status tvl_decode_greedy(tvl_model* m, int32_t start_token, int32_t start_po
 tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t d_out, int32_t d_in,
                     void* stream);
 
-/* Weight-only 8-bit rows. The paper leaves quantization to future work
+/* Weight-only 8-bit rows (also the weight format of a model loaded with
+ * weight_bits = 8). The paper leaves quantization to future work
  * (§ Future Work: Quantization: narrow weights unpacked on the fly, for less
  * memory traffic per token); this is one reading of it. A matrix W [rows x
  * cols] becomes packed rows of 16 + cols bytes each: the float32 scale

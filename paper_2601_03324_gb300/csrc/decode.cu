@@ -27,6 +27,7 @@ struct tvl_model {
   size_t weight_bytes = 0;
   int64_t streamed_bytes = 0;
   DecodeArgs args{};
+  const void* kernel = nullptr;  // decode_kernel<false> or <true> (8-bit rows)
   int smem_bytes = 0;
   int* err_host = nullptr;  // pinned, mapped: the kernel writes its error code here too
   unsigned epoch = 1;       // tag of the next launch's first exchange (0 = never written)
@@ -115,7 +116,7 @@ tvl_status launch(tvl_model* m, int token, int pos, int n_steps, int final_token
   a.final_token = final_token;
   a.epoch0 = m->epoch;
   void* params[] = {&a};
-  TVL_CK(cudaLaunchCooperativeKernel((const void*)decode_kernel, dim3(a.G), dim3(kThreads), params,
+  TVL_CK(cudaLaunchCooperativeKernel(m->kernel, dim3(a.G), dim3(kThreads), params,
                                      (size_t)m->smem_bytes, m->stream));
   // tags wrap modulo 2^32; a stale word is never within one launch of a live tag
   m->epoch += (unsigned)n_steps * (unsigned)(kPhasesPerLayer * m->cfg.n_layers + 1);
@@ -142,6 +143,11 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   if (d % 32 != 0 || hd % 4 != 0 || hd > 128 || F % 4 != 0 || std::max(d, F) > 16384) {
     set_error("tvl_load: the GPU path needs dim % 32 == 0, head_dim % 4 == 0 and <= 128, "
               "hidden_dim % 4 == 0, max(dim, hidden_dim) <= 16384");
+    return TVL_E_UNSUPPORTED;
+  }
+  const bool q8 = cfg->weight_bits == 8;
+  if (q8 && (d % 16 != 0 || F % 16 != 0 || std::max(d, F) > 16368)) {
+    set_error("tvl_load: 8-bit rows need dim and hidden_dim multiples of 16 and at most 16368");
     return TVL_E_UNSUPPORTED;
   }
   // §5.1 weight tying: explicit, or inferred from the blob size.
@@ -176,6 +182,7 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
     return e == cudaSuccess ? TVL_OK : cuda_fail(e, what);
   };
   tvl_status st;
+  m->kernel = q8 ? (const void*)decode_kernel<true> : (const void*)decode_kernel<false>;
   if ((st = ck(cudaGetDevice(&m->device), "cudaGetDevice")) != TVL_OK) return fail(st);
   int sms = 0, coop = 0, max_optin = 0;
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, m->device);
@@ -204,12 +211,12 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
     return fail(TVL_E_UNSUPPORTED);
   }
   m->smem_bytes = sp.total;
-  if ((st = ck(cudaFuncSetAttribute((const void*)decode_kernel,
+  if ((st = ck(cudaFuncSetAttribute(m->kernel,
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, sp.total),
                "cudaFuncSetAttribute")) != TVL_OK)
     return fail(st);
   int per_sm = 0;
-  if ((st = ck(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, (const void*)decode_kernel,
+  if ((st = ck(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, m->kernel,
                                                               kThreads, sp.total),
                "cudaOccupancyMaxActiveBlocksPerMultiprocessor")) != TVL_OK)
     return fail(st);
@@ -227,6 +234,25 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
     return at;
   };
   const size_t o_w = take(blob_bytes);
+  // 8-bit rows: per layer [Wq|Wk|Wv], Wo, [W1|W3], W2; then E and the untied classifier
+  const size_t rq = 16 + (size_t)d, rf = 16 + (size_t)F;
+  size_t q_wqkv = 0, q_wo = 0, q_w13 = 0, q_w2 = 0, q_stride = 0, o_q = 0, o_qE = 0, o_qcls = 0;
+  if (q8) {
+    size_t lo = 0;
+    auto ltake = [&](size_t bytes) {
+      const size_t at = lo;
+      lo = (size_t)a256((int64_t)(lo + bytes));
+      return at;
+    };
+    q_wqkv = ltake((size_t)(d + 2 * kvd) * rq);
+    q_wo = ltake((size_t)d * rq);
+    q_w13 = ltake((size_t)2 * F * rq);
+    q_w2 = ltake((size_t)d * rf);
+    q_stride = lo;
+    o_q = take(q_stride * (size_t)L);
+    o_qE = take((size_t)V * rq);
+    o_qcls = tied ? o_qE : take((size_t)V * rq);
+  }
   const size_t o_rope = take((size_t)S * (hd / 2) * sizeof(float2));
   const size_t kv_bytes = (size_t)std::max(L, 1) * S * kvd * 4;
   const size_t o_kc = take(kv_bytes), o_vc = take(kv_bytes);
@@ -284,6 +310,25 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   if (st == TVL_OK) st = ck(cudaStreamSynchronize(m->stream), "cudaStreamSynchronize(blob)");
   if (registered) cudaHostUnregister(const_cast<void*>(blob));
   if (st != TVL_OK) return fail(st);
+  if (q8) {  // every weight matrix to 8-bit rows, on the device (tvl_quantize_q8)
+    const unsigned char* Wf = m->arena + o_w;
+    auto quant = [&](const unsigned char* src, size_t dst, int rows, int cols) {
+      return tvl_quantize_q8(reinterpret_cast<const float*>(src), m->arena + dst, rows, cols,
+                             m->stream);
+    };
+    for (int l = 0; l < L && st == TVL_OK; ++l) {
+      const unsigned char* lw = Wf + bl.l0 + (size_t)l * bl.stride;
+      const size_t ql = o_q + (size_t)l * q_stride;
+      st = quant(lw + bl.wq, ql + q_wqkv, d + 2 * kvd, d);
+      if (st == TVL_OK) st = quant(lw + bl.wo, ql + q_wo, d, d);
+      if (st == TVL_OK) st = quant(lw + bl.w1, ql + q_w13, 2 * F, d);
+      if (st == TVL_OK) st = quant(lw + bl.w2, ql + q_w2, d, F);
+    }
+    if (st == TVL_OK) st = quant(Wf + bl.E, o_qE, V, d);
+    if (st == TVL_OK && !tied) st = quant(Wf + bl.Wcls, o_qcls, V, d);
+    if (st == TVL_OK) st = ck(cudaStreamSynchronize(m->stream), "cudaStreamSynchronize(q8)");
+    if (st != TVL_OK) return fail(st);
+  }
 
   // ---- RoPE table: pair i at position p turns by p * theta^(-2i/hd) ------------------
   {
@@ -319,6 +364,14 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   a.o_gffn = bl.g_ffn;
   a.o_w13 = bl.w1;
   a.o_w2 = bl.w2;
+  a.q_layer0 = q8 ? m->arena + o_q : nullptr;
+  a.q_stride = (long long)q_stride;
+  a.q_wqkv = (long long)q_wqkv;
+  a.q_wo = (long long)q_wo;
+  a.q_w13 = (long long)q_w13;
+  a.q_w2 = (long long)q_w2;
+  a.q_E = q8 ? m->arena + o_qE : nullptr;
+  a.q_cls = q8 ? m->arena + o_qcls : nullptr;
   a.rope = reinterpret_cast<const float2*>(m->arena + o_rope);
   a.kc = reinterpret_cast<float*>(m->arena + o_kc);
   a.vc = reinterpret_cast<float*>(m->arena + o_vc);
@@ -345,8 +398,11 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   a.sm_seg = sp.seg; a.sm_att = sp.att; a.sm_misc = sp.misc;
   a.wait_limit_ns = kWaitLimitNs;
   m->streamed_bytes =
-      4LL * ((int64_t)L * ((int64_t)(d + 2 * kvd) * d + (int64_t)d * d + 3LL * F * d + 2LL * d) +
-             (int64_t)V * d + 2LL * d);
+      q8 ? (int64_t)L * ((int64_t)(d + 2 * kvd) * (16 + d) + (int64_t)d * (16 + d) +
+                         2LL * F * (16 + d) + (int64_t)d * (16 + F) + 8LL * d) +
+               (int64_t)V * (16 + d) + (16 + d) + 4LL * d
+         : 4LL * ((int64_t)L * ((int64_t)(d + 2 * kvd) * d + (int64_t)d * d + 3LL * F * d + 2LL * d) +
+                  (int64_t)V * d + 2LL * d);
   *out = m;
   return TVL_OK;
 }

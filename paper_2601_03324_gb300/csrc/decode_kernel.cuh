@@ -42,6 +42,12 @@ struct DecodeArgs {
   const float* g_final;
   const float* Wcls;
   const unsigned char* layer0;
+  // 8-bit rows (models loaded with weight_bits 8): per layer [Wq|Wk|Wv], Wo,
+  // [W1|W3], W2 at these byte offsets; the embedding table; the classifier
+  const unsigned char* q_layer0;
+  long long q_stride, q_wqkv, q_wo, q_w13, q_w2;
+  const unsigned char* q_E;
+  const unsigned char* q_cls;
   long long layer_stride;  // bytes between consecutive layers
   long long o_gatt, o_wqkv, o_wo, o_gffn, o_w13, o_w2;  // byte offsets in a layer
   const float2* rope;  // [S][hd/2] (cos, sin)
@@ -614,6 +620,7 @@ __device__ inline bool reduce_candidates(const DecodeArgs& a, int parity, unsign
 
 // The weight stream of one launch, in consumption order: per step, each
 // layer's [Wq|Wk|Wv], Wo, [W1|W3], W2, then the classifier; this CTA's rows.
+template <bool kQ8>
 struct DecodeSched {
   const DecodeArgs* a;
   uint32_t refill_delay_ns = kRefillDelayNs;
@@ -623,18 +630,20 @@ struct DecodeSched {
     const int c = blockIdx.x;
     if (l < a->L) {
       const unsigned char* lw = a->layer0 + (size_t)l * a->layer_stride;
+      const unsigned char* ql = kQ8 ? a->q_layer0 + (size_t)l * a->q_stride : nullptr;
+      // 8-bit rows are 4 + K/4 words in the stages
       if (k == 0) {
-        W = reinterpret_cast<const float*>(lw + a->o_wqkv);
-        p = plan_stages(a->d + 2 * a->kvd, a->d, a->G, c);
+        W = reinterpret_cast<const float*>(kQ8 ? ql + a->q_wqkv : lw + a->o_wqkv);
+        p = plan_stages(a->d + 2 * a->kvd, kQ8 ? 4 + a->d / 4 : a->d, a->G, c);
       } else if (k == 1) {
-        W = reinterpret_cast<const float*>(lw + a->o_wo);
-        p = plan_stages(a->d, a->d, a->G, c);
+        W = reinterpret_cast<const float*>(kQ8 ? ql + a->q_wo : lw + a->o_wo);
+        p = plan_stages(a->d, kQ8 ? 4 + a->d / 4 : a->d, a->G, c);
       } else if (k == 2) {
-        W = reinterpret_cast<const float*>(lw + a->o_w13);
-        p = plan_stages(2 * a->F, a->d, a->G, c);
+        W = reinterpret_cast<const float*>(kQ8 ? ql + a->q_w13 : lw + a->o_w13);
+        p = plan_stages(2 * a->F, kQ8 ? 4 + a->d / 4 : a->d, a->G, c);
       } else {
-        W = reinterpret_cast<const float*>(lw + a->o_w2);
-        p = plan_stages(a->d, a->F, a->G, c);
+        W = reinterpret_cast<const float*>(kQ8 ? ql + a->q_w2 : lw + a->o_w2);
+        p = plan_stages(a->d, kQ8 ? 4 + a->F / 4 : a->F, a->G, c);
       }
       if (++k == 4) {
         k = 0;
@@ -642,8 +651,8 @@ struct DecodeSched {
       }
       return true;
     }
-    W = a->Wcls;
-    p = plan_stages(a->V, a->d, a->G, c);
+    W = kQ8 ? reinterpret_cast<const float*>(a->q_cls) : a->Wcls;
+    p = plan_stages(a->V, kQ8 ? 4 + a->d / 4 : a->d, a->G, c);
     l = 0;
     k = 0;
     ++s;
@@ -651,6 +660,7 @@ struct DecodeSched {
   }
 };
 
+template <bool kQ8>
 __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned char* smem,
                                     volatile int* s_abort) {
   float* xs = reinterpret_cast<float*>(smem + a.sm_xs);
@@ -690,9 +700,22 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
     // barrier below order every later row load of the CTA after them.
     if (tid == 0) __threadfence();
     // x = E[token] (paper §4.1: weights are rows at offsets in the blob)
-    const float4* e4 = reinterpret_cast<const float4*>(a.E + (size_t)token * a.d);
-    for (int j = tid; j < (a.d >> 2); j += kConsumerThreads)
-      reinterpret_cast<float4*>(xs)[j] = __ldg(e4 + j);
+    if (kQ8) {  // the row the codes stand for: scale * code
+      const unsigned char* er = a.q_E + (size_t)token * (16 + a.d);
+      const float sc = __ldg(reinterpret_cast<const float*>(er));
+      const int* cw = reinterpret_cast<const int*>(er + 16);
+      for (int j = tid; j < (a.d >> 2); j += kConsumerThreads) {
+        const int w = __ldg(cw + j);
+        reinterpret_cast<float4*>(xs)[j] =
+            make_float4(sc * (float)(int)(signed char)(w & 0xff),
+                        sc * (float)(int)(signed char)((w >> 8) & 0xff),
+                        sc * (float)(int)(signed char)((w >> 16) & 0xff), sc * (float)(w >> 24));
+      }
+    } else {
+      const float4* e4 = reinterpret_cast<const float4*>(a.E + (size_t)token * a.d);
+      for (int j = tid; j < (a.d >> 2); j += kConsumerThreads)
+        reinterpret_cast<float4*>(xs)[j] = __ldg(e4 + j);
+    }
     named_bar_sync(kBarConsumers, kConsumerThreads);
     // The four GEMV phases of a layer run one copy of the phase code, in a
     // loop that is not unrolled, so the code stays in the instruction cache
@@ -736,8 +759,8 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
         const int K = k == 3 ? a.F : a.d;
         unsigned long long* out = k == 0 ? a.x_qkv : k == 1 ? a.x_o : k == 2 ? a.x_h13 : a.x_f;
         EpiTag e{out, el + (k == 0 ? 0u : (unsigned)k + 1u)};
-        if (!consume_phase<false>(r, g, plan_stages(M, K, a.G, c), vec, 1, K, seg, e, a.err,
-                                  a.err_host, s_abort))
+        if (!consume_phase<false, kQ8>(r, g, plan_stages(M, kQ8 ? 4 + K / 4 : K, a.G, c), vec, 1,
+                                       K, seg, e, a.err, a.err_host, s_abort))
           return false;
       }
     }
@@ -753,8 +776,8 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
       rmsnorm_finish(vec, xs, gp, a.g_final, a.d, a.eps, ss, red);
     }
     EpiArgmax ea{a.logits, -INFINITY, 0x7fffffff};
-    if (!consume_phase<false>(r, g, plan_stages(a.V, a.d, a.G, c), vec, 1, a.d, seg, ea, a.err,
-                       a.err_host, s_abort))
+    if (!consume_phase<false, kQ8>(r, g, plan_stages(a.V, kQ8 ? 4 + a.d / 4 : a.d, a.G, c), vec,
+                                   1, a.d, seg, ea, a.err, a.err_host, s_abort))
       return false;
     float bv = ea.bv;
     int bi = ea.bi;
@@ -778,6 +801,7 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
   return true;
 }
 
+template <bool kQ8>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_constant__ DecodeArgs a) {
   extern __shared__ __align__(128) unsigned char smem[];
   Ring r;
@@ -799,13 +823,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
   __syncthreads();
   if (threadIdx.x >= kConsumerThreads) {
     if (threadIdx.x == kConsumerThreads) {
-      DecodeSched sched;
+      DecodeSched<kQ8> sched;
       sched.a = &a;
       run_producer(r, sched, a.err, a.err_host, s_abort);
     }
     return;
   }
-  decode_steps(a, r, smem, s_abort);
+  decode_steps<kQ8>(a, r, smem, s_abort);
 }
 
 // Failure-detection self-test: one CTA polls a tagged word that nothing

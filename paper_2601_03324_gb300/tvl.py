@@ -31,7 +31,7 @@ class Config(ctypes.Structure):
         ("n_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
         ("vocab_size", ctypes.c_int32), ("max_seq", ctypes.c_int32),
         ("rope_theta", ctypes.c_double), ("norm_eps", ctypes.c_double),
-        ("shared_classifier", ctypes.c_int32),
+        ("shared_classifier", ctypes.c_int32), ("weight_bits", ctypes.c_int32),
     ]
 
 
@@ -115,7 +115,7 @@ def make_config(cfg: dict) -> Config:
         int(cfg["dim"]), int(cfg["hidden_dim"]), int(cfg["n_layers"]), int(cfg["n_heads"]),
         int(cfg["n_kv_heads"]), int(cfg["vocab_size"]), int(cfg["max_seq"]),
         float(cfg.get("rope_theta", 10000.0)), float(cfg.get("norm_eps", 1e-5)),
-        int(cfg.get("shared_classifier", 0)),
+        int(cfg.get("shared_classifier", 0)), int(cfg.get("weight_bits", 0)),
     )
 
 
