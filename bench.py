@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--warmup", type=int, default=256)
     ap.add_argument("--impl", default="tvl", choices=["tvl", "reference"])
     ap.add_argument("--workload", default="110m", choices=["110m", "110m-long", "tiny", "7b"])
+    ap.add_argument("--weights", default="f32", choices=["f32", "q8"],
+                    help="q8: weight-only 8-bit rows (tvl_config.weight_bits = 8)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
@@ -172,11 +174,11 @@ class Clocks:
                 "reasons": reasons, "samples": len(win)}
 
 
-def cpu_oracle_rate(cfg, blob, seconds: float):
+def cpu_oracle_rate(cfg, blob, seconds: float, weight_bits: int = 0):
     """The CPU oracle (double accumulators, one thread) decoding greedily from
     token 1 for about `seconds`; tokens/s."""
     import oracle
-    m = oracle.Model(cfg, blob, 64)
+    m = oracle.Model(cfg, blob, 64, weight_bits=weight_bits)
     t, n = 1, 0
     t0 = time.perf_counter()
     while True:
@@ -316,6 +318,8 @@ def main():
     from paper_2601_03324_gb300 import tvl
 
     blob = synth.make_blob(cfg)
+    if args.weights == "q8":
+        cfg = dict(cfg, weight_bits=8)
     stream = torch.cuda.Stream()
     model = tvl.Model(cfg, blob, stream=stream.cuda_stream)
     info = model.info()
@@ -382,7 +386,8 @@ def main():
     bytes_launch = sum(step_bytes(cfg, info.streamed_bytes, pos0 + p) for p in range(n_typ))
     peak, peak_src = measured_peaks()
     achieved = bytes_launch / (statistics.mean(t for t, n in full if n == n_typ) * 1e-3) / 1e9
-    traffic = committed_traffic(args.workload, bytes_launch)
+    traffic = committed_traffic(args.workload + ("_q8" if args.weights == "q8" else ""),
+                                bytes_launch)
     steps_ns = model.step_times(n_typ).astype(np.float64)
     dts = np.diff(steps_ns) / 1e3 if n_typ > 1 else np.array([launch_ms * 1e3])
 
@@ -412,7 +417,8 @@ def main():
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline and args.workload in ("110m", "tiny"):
-        rate, n, el = cpu_oracle_rate(cfg, blob, args.cpu_seconds)
+        rate, n, el = cpu_oracle_rate(cfg, blob, args.cpu_seconds,
+                                      8 if args.weights == "q8" else 0)
         cpu = {"value": rate, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                "sample": f"first {n} greedy steps of the workload from token 1 "
                          f"({el:.1f} s, double accumulators, one thread)"}
@@ -422,9 +428,10 @@ def main():
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": el_ms / args.steps,
         "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": value / PAPER_TOKS if args.workload == "110m" else None,
-        "dtype": "f32", "data": "synthetic (seeded N(0, 0.02) weights)",
-        "config": workload_config(args.workload, cfg),
+        "vs_baseline": value / PAPER_TOKS if args.workload == "110m" and args.weights == "f32" else None,
+        "dtype": "f32" if args.weights == "f32" else "f32 activations, int8 weight rows",
+        "data": "synthetic (seeded N(0, 0.02) weights)",
+        "config": dict(workload_config(args.workload, cfg), weights=args.weights),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "kernel": "decode_kernel", "peak_source": peak_src,
