@@ -270,21 +270,32 @@ def gemv_sweep(args):
     out = []
     for i, (M, K) in enumerate(synth.GEMV_SHAPES):
         W, x = synth.gemv_operands(M, K, i)
-        nbytes = 4 * (M * K + M + K)
-        copies = max(1, math.ceil(3 * l2 / (4 * M * K)))
-        dW = torch.from_numpy(W).cuda().repeat(copies, 1).reshape(copies, M, K)
+        q8 = args.weights == "q8"
+        wbytes = tvl.tvl_q8_bytes(M, K) if q8 else 4 * M * K
+        nbytes = wbytes + 4 * (M + K)
+        copies = max(1, math.ceil(3 * l2 / wbytes))
+        if q8:  # packed 8-bit rows of W, one copy per rotation slot
+            dW1 = torch.from_numpy(W).cuda()
+            dW = torch.empty((copies, wbytes), dtype=torch.uint8, device="cuda")
+            for c in range(copies):
+                tvl.tvl_quantize_q8(dW1.data_ptr(), dW[c].data_ptr(), M, K)
+            torch.cuda.synchronize()
+            del dW1
+            call = tvl.tvl_gemv_q8
+        else:
+            dW = torch.from_numpy(W).cuda().repeat(copies, 1).reshape(copies, M, K)
+            call = tvl.tvl_gemv
         dx = torch.from_numpy(x).cuda()
         dy = torch.empty(M, device="cuda")
         reps = 200
         with torch.cuda.stream(s):
             for r in range(10):
-                tvl.tvl_gemv(dW[r % copies].data_ptr(), dx.data_ptr(), dy.data_ptr(), M, K,
-                             s.cuda_stream)
+                call(dW[r % copies].data_ptr(), dx.data_ptr(), dy.data_ptr(), M, K, s.cuda_stream)
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g, stream=s):
                 for r in range(reps):
-                    tvl.tvl_gemv(dW[r % copies].data_ptr(), dx.data_ptr(), dy.data_ptr(), M, K,
-                                 s.cuda_stream)
+                    call(dW[r % copies].data_ptr(), dx.data_ptr(), dy.data_ptr(), M, K,
+                         s.cuda_stream)
             g.replay()
             s.synchronize()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -298,7 +309,8 @@ def gemv_sweep(args):
     peak, src = measured_peaks()
     for o in out:
         o["frac_of_" + src + "_hbm"] = o["GB/s"] / peak
-    print(json.dumps({"gemv_sweep": out, "peak_gbs": peak, "peak_source": src}), flush=True)
+    print(json.dumps({"gemv_sweep": out, "weights": args.weights, "peak_gbs": peak,
+                      "peak_source": src}), flush=True)
 
 
 def main():

@@ -293,10 +293,18 @@ __device__ __forceinline__ float row_partial_xr(const float4* w4, const float4 (
 // stage a row is Kw = 4 + K/4 words. Code word e holds codes 4e..4e+3 and
 // meets x float4 e.
 __device__ __forceinline__ void fma_codes(float4& acc, int w, const float4& x) {
-  acc.x = fmaf((float)(int)(signed char)(w & 0xff), x.x, acc.x);
-  acc.y = fmaf((float)(int)(signed char)((w >> 8) & 0xff), x.y, acc.y);
-  acc.z = fmaf((float)(int)(signed char)((w >> 16) & 0xff), x.z, acc.z);
-  acc.w = fmaf((float)(w >> 24), x.w, acc.w);
+  // code + 128 as the low byte of the float 2^23 + (code + 128): one byte
+  // permute and one exact subtraction per code, on full-rate pipes (an
+  // integer-to-float conversion is a quarter-rate instruction)
+  const unsigned u = (unsigned)w ^ 0x80808080u;
+  const float c0 = __uint_as_float(__byte_perm(u, 0x4B000000u, 0x7540)) - 8388736.0f;
+  const float c1 = __uint_as_float(__byte_perm(u, 0x4B000000u, 0x7541)) - 8388736.0f;
+  const float c2 = __uint_as_float(__byte_perm(u, 0x4B000000u, 0x7542)) - 8388736.0f;
+  const float c3 = __uint_as_float(__byte_perm(u, 0x4B000000u, 0x7543)) - 8388736.0f;
+  acc.x = fmaf(c0, x.x, acc.x);
+  acc.y = fmaf(c1, x.y, acc.y);
+  acc.z = fmaf(c2, x.z, acc.z);
+  acc.w = fmaf(c3, x.w, acc.w);
 }
 
 // Lane partials of sum_j q_j x_j for two 8-bit rows sharing x (nw code words).
