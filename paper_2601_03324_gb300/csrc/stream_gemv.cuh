@@ -311,7 +311,7 @@ __device__ __forceinline__ void fma_codes(float4& acc, int w, const float4& x) {
 __device__ __forceinline__ float2 row2_partial_q8(const int* c0, const int* c1, const float4* x4,
                                                   int nw, int lane) {
   float4 a = make_float4(0.f, 0.f, 0.f, 0.f), b = a;
-#pragma unroll 2
+#pragma unroll 8
   for (int e = lane; e < nw; e += 32) {
     const float4 x = x4[e];
     fma_codes(a, c0[e], x);
@@ -322,7 +322,7 @@ __device__ __forceinline__ float2 row2_partial_q8(const int* c0, const int* c1, 
 
 __device__ __forceinline__ float row_partial_q8(const int* c0, const float4* x4, int nw, int lane) {
   float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 2
+#pragma unroll 8
   for (int e = lane; e < nw; e += 32) fma_codes(a, c0[e], x4[e]);
   return (a.x + a.y) + (a.z + a.w);
 }
