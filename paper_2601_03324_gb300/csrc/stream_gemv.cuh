@@ -335,6 +335,9 @@ __device__ inline bool warp_wait_full(const Ring& r, int slot, uint32_t gs, int*
                                       int* err_host, volatile int* s_abort) {
   uint64_t* bar = &r.full[slot];
   const uint32_t par = (gs / (uint32_t)r.nst) & 1u;
+  // usual case: the stage was queued long ago and has landed
+  if (__all_sync(0xffffffffu, r.seq[slot] == (int)(gs + 1u) && mbar_test_wait(bar, par)))
+    return true;
   bool ok = true;
   if (r.seq[slot] != (int)(gs + 1u)) {
     const bool leader = (threadIdx.x & 31) == 0;
