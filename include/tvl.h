@@ -54,6 +54,9 @@ typedef struct {
                            matrix (and the embedding table) into 8-bit rows, as
                            tvl_quantize_q8 defines, and decodes with them; dim and
                            hidden_dim must then be multiples of 16 */
+  int32_t max_batch;    /* sequences one launch may decode together, 0 or 1 (one) to 4;
+                           each sequence slot gets its own KV cache and exchange buffers.
+                           More than one needs weight_bits 0 */
 } tvl_config;
 
 typedef struct tvl_model tvl_model; /* opaque: device arena, stream, kernel plan */
@@ -111,6 +114,29 @@ tvl_status tvl_forward(tvl_model* m, int32_t token, int32_t pos, float* logits_o
  *   start_pos + n_steps <= max_seq, n_steps >= 1, else TVL_E_RANGE. */
 tvl_status tvl_decode_greedy(tvl_model* m, int32_t start_token, int32_t start_pos,
                              int32_t n_steps, int32_t* tokens_out);
+
+/* Batched decode: `batch` independent sequences (1 <= batch <= max_batch,
+ * else TVL_E_INVAL) advance together, one position per step, in one kernel
+ * launch that streams every weight once per step for all of them. The paper
+ * (§ Implications for Computational Linguistics, "Enabling Advanced Decoding
+ * Strategies") names beam search with B = 4 hypotheses as the case whose
+ * bandwidth need grows B-fold when each hypothesis is decoded on its own;
+ * here the B hypotheses share each step's single weight stream. Sequence b uses KV-cache slot b (slot 0
+ * is the cache tvl_forward and tvl_decode_greedy use); all sequences are at
+ * the same position pos and must have written positions 0..pos-1 of their
+ * slots. Results per sequence equal a separate batch-1 run up to float
+ * rounding (sums are taken in another order).
+ * tvl_forward_batch: one step; tokens[b] (host array of batch) at position
+ *   pos; logits_out [batch][V] (device pointer: queued, no wait; host: waits
+ *   and reports device errors; NULL: kept on the device).
+ * tvl_decode_greedy_batch: n_steps greedy steps from start_tokens[b] at
+ *   start_pos; tokens_out (host, NULL allowed) [n_steps][batch]:
+ *   tokens_out[s * batch + b] = argmax of sequence b's logits after step s.
+ * Token out of range, pos < 0 or start_pos + n_steps > max_seq: TVL_E_RANGE. */
+tvl_status tvl_forward_batch(tvl_model* m, int32_t batch, const int32_t* tokens, int32_t pos,
+                             float* logits_out);
+tvl_status tvl_decode_greedy_batch(tvl_model* m, int32_t batch, const int32_t* start_tokens,
+                                   int32_t start_pos, int32_t n_steps, int32_t* tokens_out);
 
 /* Standalone GEMV y = W x (§6.1), W [d_out x d_in] row-major, x [d_in],
  * y [d_out]; all device pointers; queued on `stream` (NULL = default stream),
@@ -190,6 +216,7 @@ typedef struct {
   int32_t stage_bytes;
   int32_t tied;
   int32_t barriers_per_step; /* grid-wide barriers in one greedy step */
+  int32_t max_batch;         /* as loaded (1 when the config said 0) */
 } tvl_model_info;
 tvl_status tvl_get_info(const tvl_model* m, tvl_model_info* out);
 

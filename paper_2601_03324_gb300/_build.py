@@ -16,7 +16,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 OUT = os.path.join(HERE, "libtvl.so")
 BUILD_DIR = os.path.join(HERE, "_build")
-SOURCES = ["abi.cu", "decode.cu", "gemv.cu"]
+SOURCES = ["abi.cu", "decode.cu", "decode_batch.cu", "gemv.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -27,12 +27,36 @@ struct tvl_model {
   size_t weight_bytes = 0;
   int64_t streamed_bytes = 0;
   DecodeArgs args{};
-  const void* kernel = nullptr;  // decode_kernel<false> or <true> (8-bit rows)
+  int max_batch = 1;
+  // per batch size B = 1..max_batch: the kernel (decode_kernel<q8, B>), its
+  // shared-memory plan and the words between two sequences' phase inputs
+  const void* kernel[kMaxBatch + 1] = {};
+  struct Plan {
+    int sm_ring, sm_bars, sm_xs, sm_vec, sm_seg, sm_att, sm_misc, nst, total;
+  } plan[kMaxBatch + 1] = {};
+  int vs = 0;
   int smem_bytes = 0;
   int* err_host = nullptr;  // pinned, mapped: the kernel writes its error code here too
   unsigned epoch = 1;       // tag of the next launch's first exchange (0 = never written)
   tvl_status sticky = TVL_OK;
 };
+
+namespace tvl {
+
+// Failure-detection self-test: one CTA polls a tagged word that nothing
+// writes; the bounded wait must expire and report TVL_E_TIMEOUT.
+__global__ void wait_selftest_kernel(unsigned long long* word, int* err,
+                                     unsigned long long limit_ns) {
+  __shared__ int s_abort;
+  if (threadIdx.x == 0) s_abort = 0;
+  __syncthreads();
+  if (threadIdx.x >= kConsumerThreads) return;  // the consumer warps take part
+  const Poll pc{err, nullptr, &s_abort, limit_ns};
+  const bool ok = poll_pairs(word, 1, 1u, pc, [](int, float, float) {});
+  vote_ok(ok, &s_abort);
+}
+
+}  // namespace tvl
 
 namespace {
 
@@ -40,12 +64,14 @@ struct SmemPlan {
   int ring, bars, xs, vec, seg, att, misc, total, nst;
 };
 
-SmemPlan plan_smem(int d, int F, int hd, int H, int nch_cap, int max_bytes) {
+// Shared memory of one CTA for B sequences: the ring takes what the other
+// regions leave, up to kMaxStages stages.
+SmemPlan plan_smem(int d, int F, int hd, int H, int nch_cap, int max_bytes, int B) {
   SmemPlan p{};
   const int att_floats = 3 * hd + kAttMaxChunk + 4 * kConsumerThreads + nch_cap * (hd + 2) + 16;
   // every region is a multiple of 128 bytes, so every region starts aligned
-  const int xs = (int)a128(4LL * d), vec = (int)a128(4LL * std::max(d, F));
-  const int seg = (int)a128(kMaxSegParts * 4), att = (int)a128(4LL * att_floats), misc = 256;
+  const int xs = (int)a128(4LL * B * d), vec = (int)a128(4LL * B * std::max(d, F));
+  const int seg = (int)a128(kMaxSegParts * 4), att = (int)a128(4LL * att_floats), misc = 512;
   const int bars = (int)a128(kRingBarBytes);
   const int other = bars + xs + vec + seg + att + misc;
   int nst = (max_bytes - other) / kStageBytes;
@@ -108,16 +134,22 @@ bool is_device_pointer(const void* p) {
   return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
 }
 
-tvl_status launch(tvl_model* m, int token, int pos, int n_steps, int final_token) {
+tvl_status launch(tvl_model* m, int B, const int* tokens, int pos, int n_steps,
+                  int final_token) {
   DecodeArgs a = m->args;
-  a.start_token = token;
+  for (int b = 0; b < B; ++b) a.start_tokens[b] = tokens[b];
   a.start_pos = pos;
   a.n_steps = n_steps;
   a.final_token = final_token;
   a.epoch0 = m->epoch;
+  const tvl_model::Plan& pl = m->plan[B];
+  a.nst = pl.nst;
+  a.sm_ring = pl.sm_ring; a.sm_bars = pl.sm_bars; a.sm_xs = pl.sm_xs; a.sm_vec = pl.sm_vec;
+  a.sm_seg = pl.sm_seg; a.sm_att = pl.sm_att; a.sm_misc = pl.sm_misc;
+  a.vs = m->vs;
   void* params[] = {&a};
-  TVL_CK(cudaLaunchCooperativeKernel(m->kernel, dim3(a.G), dim3(kThreads), params,
-                                     (size_t)m->smem_bytes, m->stream));
+  TVL_CK(cudaLaunchCooperativeKernel(m->kernel[B], dim3(a.G), dim3(kThreads), params,
+                                     (size_t)pl.total, m->stream));
   // tags wrap modulo 2^32; a stale word is never within one launch of a live tag
   m->epoch += (unsigned)n_steps * (unsigned)(kPhasesPerLayer * m->cfg.n_layers + 1);
   return TVL_OK;
@@ -146,6 +178,11 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
     return TVL_E_UNSUPPORTED;
   }
   const bool q8 = cfg->weight_bits == 8;
+  const int maxB = cfg->max_batch > 1 ? cfg->max_batch : 1;
+  if (maxB > 1 && q8) {
+    set_error("tvl_load: max_batch > 1 needs float32 weights (weight_bits 0)");
+    return TVL_E_UNSUPPORTED;
+  }
   if (q8 && (d % 16 != 0 || F % 16 != 0 || std::max(d, F) > 16368)) {
     set_error("tvl_load: 8-bit rows need dim and hidden_dim multiples of 16 and at most 16368");
     return TVL_E_UNSUPPORTED;
@@ -174,6 +211,7 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   if (!m) return TVL_E_NOMEM;
   m->cfg = *cfg;
   m->tied = tied;
+  m->max_batch = maxB;
   auto fail = [&](tvl_status s) {
     destroy(m);
     return s;
@@ -182,7 +220,8 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
     return e == cudaSuccess ? TVL_OK : cuda_fail(e, what);
   };
   tvl_status st;
-  m->kernel = q8 ? (const void*)decode_kernel<true> : (const void*)decode_kernel<false>;
+  m->kernel[1] = q8 ? (const void*)decode_kernel<true, 1> : (const void*)decode_kernel<false, 1>;
+  for (int B = 2; B <= maxB; ++B) m->kernel[B] = decode_kernel_for_batch(B);
   if ((st = ck(cudaGetDevice(&m->device), "cudaGetDevice")) != TVL_OK) return fail(st);
   int sms = 0, coop = 0, max_optin = 0;
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, m->device);
@@ -193,37 +232,45 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
     return fail(TVL_E_UNSUPPORTED);
   }
   const int G = sms;
+  // a head gets the most attention chunks with one sequence: this bounds every B
   const int nch_cap = nch_cap_for(S, H, G);
-  const SmemPlan sp = plan_smem(d, F, hd, H, nch_cap, max_optin);
-  {  // segment partials of rows longer than a stage must fit the scratch
-    const long long Ms[5] = {d + 2LL * kvd, d, 2LL * F, d, V};
-    const int Ks[5] = {d, d, d, F, d};
-    for (int i = 0; i < 5; ++i) {
-      const StagePlan pl = plan_stages(Ms[i], Ks[i], G, 0);
-      if (pl.spr > 1 && (long long)((Ms[i] + G - 1) / G) * pl.spr > kMaxSegParts) {
-        set_error("tvl_load: too many long rows per SM for the segment scratch");
-        return fail(TVL_E_UNSUPPORTED);
+  for (int B = 1; B <= maxB; ++B) {
+    const SmemPlan sp = plan_smem(d, F, hd, H, nch_cap, max_optin, B);
+    {  // segment partials of rows longer than a stage must fit the scratch
+      const long long Ms[5] = {d + 2LL * kvd, d, 2LL * F, d, V};
+      const int Ks[5] = {d, d, d, F, d};
+      for (int i = 0; i < 5; ++i) {
+        const StagePlan pl = plan_stages(Ms[i], Ks[i], G, 0);
+        if (pl.spr > 1 && (long long)((Ms[i] + G - 1) / G) * pl.spr * B > kMaxSegParts) {
+          set_error("tvl_load: too many long rows per SM for the segment scratch");
+          return fail(TVL_E_UNSUPPORTED);
+        }
       }
     }
+    // two stages at least; with several sequences four, or the stream stalls
+    if (sp.nst < (B == 1 ? 2 : 4)) {
+      set_error("tvl_load: not enough shared memory for the weight stages with " +
+                std::to_string(B) + " sequence(s); lower max_batch");
+      return fail(TVL_E_UNSUPPORTED);
+    }
+    if ((st = ck(cudaFuncSetAttribute(m->kernel[B],
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, sp.total),
+                 "cudaFuncSetAttribute")) != TVL_OK)
+      return fail(st);
+    int per_sm = 0;
+    if ((st = ck(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, m->kernel[B],
+                                                                kThreads, sp.total),
+                 "cudaOccupancyMaxActiveBlocksPerMultiprocessor")) != TVL_OK)
+      return fail(st);
+    if (per_sm < 1) {
+      set_error("tvl_load: decode kernel cannot be resident on an SM");
+      return fail(TVL_E_UNSUPPORTED);
+    }
+    m->plan[B] = tvl_model::Plan{sp.ring, sp.bars, sp.xs, sp.vec, sp.seg, sp.att, sp.misc,
+                                 sp.nst, sp.total};
   }
-  if (sp.nst < 2) {
-    set_error("tvl_load: not enough shared memory for two weight stages");
-    return fail(TVL_E_UNSUPPORTED);
-  }
-  m->smem_bytes = sp.total;
-  if ((st = ck(cudaFuncSetAttribute(m->kernel,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, sp.total),
-               "cudaFuncSetAttribute")) != TVL_OK)
-    return fail(st);
-  int per_sm = 0;
-  if ((st = ck(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, m->kernel,
-                                                              kThreads, sp.total),
-               "cudaOccupancyMaxActiveBlocksPerMultiprocessor")) != TVL_OK)
-    return fail(st);
-  if (per_sm < 1) {
-    set_error("tvl_load: decode kernel cannot be resident on an SM");
-    return fail(TVL_E_UNSUPPORTED);
-  }
+  m->smem_bytes = m->plan[1].total;
+  m->vs = std::max(d, F);
 
   // ---- arena: weights | rope | K cache | V cache | scratch -------------------------
   const int att_stride = hd + 4;
@@ -254,14 +301,18 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
     o_qcls = tied ? o_qE : take((size_t)V * rq);
   }
   const size_t o_rope = take((size_t)S * (hd / 2) * sizeof(float2));
-  const size_t kv_bytes = (size_t)std::max(L, 1) * S * kvd * 4;
+  // K/V cache and exchange buffers: one of each per sequence slot
+  const size_t kv_seq = (size_t)std::max(L, 1) * S * kvd;  // floats per sequence
+  const size_t kv_bytes = kv_seq * 4 * maxB;
   const size_t o_kc = take(kv_bytes), o_vc = take(kv_bytes);
   const size_t o_scr = off;
-  const size_t o_qkv = take(8ull * (d + 2 * kvd)), o_o = take(8ull * d), o_h13 = take(16ull * F);
-  const size_t o_f = take(8ull * d), o_lg = take(4ull * V);
-  const size_t o_att = take(8ull * H * nch_cap * att_stride);
-  const size_t o_attn = take(8ull * d);
-  const size_t o_cand = take(8ull * 2 * G * 2), o_tok = take(4ull * S);
+  const size_t nB = (size_t)maxB;
+  const size_t o_qkv = take(8ull * (d + 2 * kvd) * nB), o_o = take(8ull * d * nB);
+  const size_t o_h13 = take(16ull * F * nB);
+  const size_t o_f = take(8ull * d * nB), o_lg = take(4ull * V * nB);
+  const size_t o_att = take(8ull * H * nch_cap * att_stride * nB);
+  const size_t o_attn = take(8ull * d * nB);
+  const size_t o_cand = take(8ull * 2 * G * 2 * nB), o_tok = take(4ull * S * nB);
   const size_t o_ts = take(8ull * S), o_err = take(4);
   m->arena_bytes = off;
   m->weight_bytes = blob_bytes;
@@ -393,9 +444,7 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   a.nch_cap = nch_cap;
   a.eps = (float)cfg->norm_eps;
   a.att_scale = (float)(1.0 / std::sqrt((double)hd));
-  a.nst = sp.nst;
-  a.sm_ring = sp.ring; a.sm_bars = sp.bars; a.sm_xs = sp.xs; a.sm_vec = sp.vec;
-  a.sm_seg = sp.seg; a.sm_att = sp.att; a.sm_misc = sp.misc;
+  a.kv_seq = (long long)kv_seq;
   a.wait_limit_ns = kWaitLimitNs;
   m->streamed_bytes =
       q8 ? (int64_t)L * ((int64_t)(d + 2 * kvd) * (16 + d) + (int64_t)d * (16 + d) +
@@ -439,20 +488,30 @@ tvl_status tvl_load_file(const tvl_config* cfg, const char* path, void* stream, 
   return st;
 }
 
-tvl_status tvl_forward(tvl_model* m, int32_t token, int32_t pos, float* logits_out) {
-  if (!m) {
-    set_error("tvl_forward: null model");
+tvl_status tvl_forward_batch(tvl_model* m, int32_t batch, const int32_t* tokens, int32_t pos,
+                             float* logits_out) {
+  if (!m || !tokens) {
+    set_error("tvl_forward_batch: null argument");
     return TVL_E_INVAL;
   }
   if (m->sticky != TVL_OK) return m->sticky;
-  if (token < 0 || token >= m->cfg.vocab_size || pos < 0 || pos >= m->cfg.max_seq) {
-    set_error("tvl_forward: token or position out of range");
+  if (batch < 1 || batch > m->max_batch) {
+    set_error("tvl_forward_batch: batch must be in [1, max_batch of the model]");
+    return TVL_E_INVAL;
+  }
+  for (int b = 0; b < batch; ++b)
+    if (tokens[b] < 0 || tokens[b] >= m->cfg.vocab_size) {
+      set_error("tvl_forward_batch: token out of range");
+      return TVL_E_RANGE;
+    }
+  if (pos < 0 || pos >= m->cfg.max_seq) {
+    set_error("tvl_forward_batch: position out of range");
     return TVL_E_RANGE;
   }
-  tvl_status st = launch(m, token, pos, 1, 0);
+  tvl_status st = launch(m, batch, tokens, pos, 1, 0);
   if (st != TVL_OK) return st;
   if (!logits_out) return TVL_OK;
-  const size_t bytes = (size_t)m->cfg.vocab_size * 4;
+  const size_t bytes = (size_t)m->cfg.vocab_size * 4 * batch;
   if (is_device_pointer(logits_out)) {
     TVL_CK(cudaMemcpyAsync(logits_out, m->args.logits, bytes, cudaMemcpyDeviceToDevice,
                            m->stream));
@@ -463,25 +522,50 @@ tvl_status tvl_forward(tvl_model* m, int32_t token, int32_t pos, float* logits_o
   return check_device_error(m);
 }
 
+tvl_status tvl_forward(tvl_model* m, int32_t token, int32_t pos, float* logits_out) {
+  if (!m) {
+    set_error("tvl_forward: null model");
+    return TVL_E_INVAL;
+  }
+  return tvl_forward_batch(m, 1, &token, pos, logits_out);
+}
+
+tvl_status tvl_decode_greedy_batch(tvl_model* m, int32_t batch, const int32_t* start_tokens,
+                                   int32_t start_pos, int32_t n_steps, int32_t* tokens_out) {
+  if (!m || !start_tokens) {
+    set_error("tvl_decode_greedy_batch: null argument");
+    return TVL_E_INVAL;
+  }
+  if (m->sticky != TVL_OK) return m->sticky;
+  if (batch < 1 || batch > m->max_batch) {
+    set_error("tvl_decode_greedy_batch: batch must be in [1, max_batch of the model]");
+    return TVL_E_INVAL;
+  }
+  for (int b = 0; b < batch; ++b)
+    if (start_tokens[b] < 0 || start_tokens[b] >= m->cfg.vocab_size) {
+      set_error("tvl_decode_greedy_batch: token out of range");
+      return TVL_E_RANGE;
+    }
+  if (start_pos < 0 || n_steps < 1 || (int64_t)start_pos + n_steps > m->cfg.max_seq) {
+    set_error("tvl_decode_greedy_batch: position or step count out of range");
+    return TVL_E_RANGE;
+  }
+  tvl_status st = launch(m, batch, start_tokens, start_pos, n_steps, 1);
+  if (st != TVL_OK) return st;
+  if (!tokens_out) return TVL_OK;
+  TVL_CK(cudaMemcpyAsync(tokens_out, m->args.tokens, 4ull * n_steps * batch,
+                         cudaMemcpyDeviceToHost, m->stream));
+  TVL_CK(cudaStreamSynchronize(m->stream));
+  return check_device_error(m);
+}
+
 tvl_status tvl_decode_greedy(tvl_model* m, int32_t start_token, int32_t start_pos,
                              int32_t n_steps, int32_t* tokens_out) {
   if (!m) {
     set_error("tvl_decode_greedy: null model");
     return TVL_E_INVAL;
   }
-  if (m->sticky != TVL_OK) return m->sticky;
-  if (start_token < 0 || start_token >= m->cfg.vocab_size || start_pos < 0 || n_steps < 1 ||
-      (int64_t)start_pos + n_steps > m->cfg.max_seq) {
-    set_error("tvl_decode_greedy: token, position or step count out of range");
-    return TVL_E_RANGE;
-  }
-  tvl_status st = launch(m, start_token, start_pos, n_steps, 1);
-  if (st != TVL_OK) return st;
-  if (!tokens_out) return TVL_OK;
-  TVL_CK(cudaMemcpyAsync(tokens_out, m->args.tokens, 4ull * n_steps, cudaMemcpyDeviceToHost,
-                         m->stream));
-  TVL_CK(cudaStreamSynchronize(m->stream));
-  return check_device_error(m);
+  return tvl_decode_greedy_batch(m, 1, &start_token, start_pos, n_steps, tokens_out);
 }
 
 tvl_status tvl_sync(tvl_model* m) {
@@ -511,10 +595,11 @@ tvl_status tvl_get_info(const tvl_model* m, tvl_model_info* out) {
   out->grid = m->args.G;
   out->threads = kThreads;
   out->smem_bytes = m->smem_bytes;
-  out->ring_stages = m->args.nst;
+  out->ring_stages = m->plan[1].nst;
   out->stage_bytes = kStageBytes;
   out->tied = m->tied ? 1 : 0;
   out->barriers_per_step = kPhasesPerLayer * m->cfg.n_layers + 1;
+  out->max_batch = m->max_batch;
   return TVL_OK;
 }
 

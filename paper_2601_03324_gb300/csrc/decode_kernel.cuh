@@ -34,6 +34,7 @@ namespace tvl {
 constexpr int kAttMinChunk = 32;    // positions per attention work item, at least
 constexpr int kAttMaxChunk = 1024;  // and at most
 constexpr int kPhasesPerLayer = 5;  // exchanges per layer: qkv, att, o, h13, f
+constexpr int kMaxBatch = 4;        // sequences one launch can decode together
 constexpr uint32_t kRefillDelayNs = 1000;  // producer pause before refilling freed stages
 
 struct DecodeArgs {
@@ -71,7 +72,13 @@ struct DecodeArgs {
   int att_stride, nch_cap;
   float eps, att_scale;
   // this launch
-  int start_token, start_pos, n_steps, final_token;
+  int start_pos, n_steps, final_token;
+  // B sequences decode in lockstep at the same positions: sequence b's words
+  // in an exchange buffer sit b vector lengths in, its K/V cache b * kv_seq
+  // floats in, its logits b * V floats in; tokens are [step][B]
+  int start_tokens[kMaxBatch];
+  long long kv_seq;
+  int vs;  // floats between two sequences' phase inputs in shared memory
   unsigned epoch0;  // tag of the first exchange of this launch
   int nst;
   int sm_ring, sm_bars, sm_xs, sm_vec, sm_seg, sm_att, sm_misc;  // byte offsets
@@ -179,10 +186,11 @@ __device__ inline bool poll_pairs(const unsigned long long* src, int npairs, uns
   return true;
 }
 
-// Same, over two tagged vectors read in step: fn(p, a0, a1, b0, b1).
-template <class Fn>
-__device__ inline bool poll_pairs2(const unsigned long long* sa, const unsigned long long* sb,
-                                   int npairs, unsigned tag, const Poll& c, Fn fn) {
+// Same, over two tagged vectors read in step: the pair at addr(p) and the
+// one `off` words after it; fn(p, a0, a1, b0, b1).
+template <class Addr, class Fn>
+__device__ inline bool poll_pairs2(int npairs, Addr addr, long long off, unsigned tag,
+                                   const Poll& c, Fn fn) {
   for (int base = threadIdx.x; base < npairs; base += kConsumerThreads * 4) {
     ulonglong2 va[4], vb[4];
     unsigned pending = 0;
@@ -190,8 +198,8 @@ __device__ inline bool poll_pairs2(const unsigned long long* sa, const unsigned 
     for (int b = 0; b < 4; ++b) {
       const int p = base + b * kConsumerThreads;
       if (p < npairs) {
-        va[b] = ld_tag2(sa + 2 * p);
-        vb[b] = ld_tag2(sb + 2 * p);
+        va[b] = ld_tag2(addr(p));
+        vb[b] = ld_tag2(addr(p) + off);
         pending |= 1u << b;
       }
     }
@@ -211,8 +219,8 @@ __device__ inline bool poll_pairs2(const unsigned long long* sa, const unsigned 
       for (int b = 0; b < 4; ++b) {
         if ((pending >> b) & 1u) {
           const int p = base + b * kConsumerThreads;
-          va[b] = ld_tag2(sa + 2 * p);
-          vb[b] = ld_tag2(sb + 2 * p);
+          va[b] = ld_tag2(addr(p));
+          vb[b] = ld_tag2(addr(p) + off);
         }
       }
     }
@@ -325,6 +333,27 @@ __device__ inline void block_argmax(float& v, int& idx, float* redv, int* redi) 
   named_bar_sync(kBarConsumers, kConsumerThreads);
 }
 
+// Sums over the consumer threads of kB values at once (one barrier pair);
+// red holds 7 * kB floats. Every thread gets the totals.
+template <int kB>
+__device__ inline void block_sum_n(float (&v)[kB], float* red) {
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+#pragma unroll
+  for (int b = 0; b < kB; ++b) {
+    const float t = warp_sum(v[b]);
+    if (lane == 0) red[warp * kB + b] = t;
+  }
+  named_bar_sync(kBarConsumers, kConsumerThreads);
+#pragma unroll
+  for (int b = 0; b < kB; ++b) {
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < kConsumerWarps; ++w) t += red[w * kB + b];
+    v[b] = t;
+  }
+  named_bar_sync(kBarConsumers, kConsumerThreads);
+}
+
 // RMSNorm gains, loaded into registers ahead of use so that their loads
 // overlap the exchange that delivers x (elements 4j..4j+3 for j = tid + 224k).
 struct Gains {
@@ -363,6 +392,39 @@ __device__ inline void rmsnorm_finish(float* out, const float* x, const Gains& g
   named_bar_sync(kBarConsumers, kConsumerThreads);
 }
 
+// RMSNorm of kB vectors (x_b at x + b * n, out_b at out + b * vs) with the
+// same gains; ss[b] = this thread's share of sum x_b^2.
+template <int kB>
+__device__ inline void rmsnorm_finish_n(float* out, int vs, const float* x, const Gains& gp,
+                                        const float* g, int n, float eps, float (&ss)[kB],
+                                        float* red) {
+  if constexpr (kB == 1) {
+    rmsnorm_finish(out, x, gp, g, n, eps, ss[0], red);
+    return;
+  }
+  block_sum_n<kB>(ss, red);  // its barriers also publish x
+  const int n4 = n >> 2;
+#pragma unroll
+  for (int b = 0; b < kB; ++b) {
+    const float r = 1.0f / sqrtf(ss[b] / (float)n + eps);
+    const float4* x4 = reinterpret_cast<const float4*>(x + (size_t)b * n);
+    float4* o4 = reinterpret_cast<float4*>(out + (size_t)b * vs);
+    auto emit = [&](int j, const float4& gv) {
+      const float4 xv = x4[j];
+      o4[j] = make_float4((xv.x * gv.x) * r, (xv.y * gv.y) * r, (xv.z * gv.z) * r,
+                          (xv.w * gv.w) * r);
+    };
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int j = threadIdx.x + k * kConsumerThreads;
+      if (j < n4) emit(j, gp.v[k]);
+    }
+    for (int j = threadIdx.x + 4 * kConsumerThreads; j < n4; j += kConsumerThreads)
+      emit(j, __ldg(reinterpret_cast<const float4*>(g) + j));
+  }
+  named_bar_sync(kBarConsumers, kConsumerThreads);
+}
+
 // This thread's share of sum x^2 when no exchange delivered x.
 __device__ inline float sum_sq(const float* x, int n) {
   float ss = 0.f;
@@ -373,16 +435,31 @@ __device__ inline float sum_sq(const float* x, int n) {
 struct EpiTag {
   unsigned long long* out;
   unsigned tag;
+  int M;  // words between two sequences' outputs
   __device__ __forceinline__ void store(int row, float v) { st_tag(out + row, tag, v); }
+  __device__ __forceinline__ void store_b(int row, int b, float v) {
+    st_tag(out + (size_t)b * M + row, tag, v);
+  }
 };
 
+// Logits of every sequence (V apart) and each thread's best (value, index)
+// per sequence so far.
+template <int kB>
 struct EpiArgmax {
   float* out;
-  float bv;
-  int bi;
-  __device__ __forceinline__ void store(int row, float v) {
-    out[row] = v;
-    if (better(v, row, bv, bi)) { bv = v; bi = row; }
+  int V;
+  float bv[kB];
+  int bi[kB];
+  __device__ __forceinline__ void init() {
+#pragma unroll
+    for (int b = 0; b < kB; ++b) { bv[b] = -INFINITY; bi[b] = 0x7fffffff; }
+  }
+  __device__ __forceinline__ void store(int row, float v) { store_b(row, 0, v); }
+  __device__ __forceinline__ void store_b(int row, int b, float v) {
+    out[(size_t)b * V + row] = v;
+#pragma unroll
+    for (int bb = 0; bb < kB; ++bb)
+      if (bb == b && better(v, row, bv[bb], bi[bb])) { bv[bb] = v; bi[bb] = row; }
   }
 };
 
@@ -392,14 +469,16 @@ struct EpiArgmax {
 // items of layer l will read: the cache lines are usually no longer in L2
 // (the weight stream has gone through it since), and the request is issued a
 // phase ahead so that the items' own loads find them there.
+template <int kB>
 __device__ inline void att_prefetch_l2(const DecodeArgs& a, int l, int pos) {
   int nch, clen;
-  att_split(pos, a.H, a.G, &nch, &clen);
+  att_split(pos, a.H * kB, a.G, &nch, &clen);
   const int group = a.H / a.Hkv, hd = a.hd;
   const int lpr = (hd * 4 + 127) / 128;  // 128-byte lines per row
-  const size_t lay = (size_t)l * a.S * a.kvd;
-  for (int it = blockIdx.x; it < a.H * nch; it += a.G) {
-    const int h = it / nch, c = it - h * nch, kvh = h / group;
+  for (int it = blockIdx.x; it < kB * a.H * nch; it += a.G) {
+    const int b = kB == 1 ? 0 : it / (a.H * nch), hc = it - b * a.H * nch;
+    const int h = hc / nch, c = hc - h * nch, kvh = h / group;
+    const size_t lay = (size_t)b * a.kv_seq + (size_t)l * a.S * a.kvd;
     const int t0 = c * clen, te = (t0 + clen < pos) ? t0 + clen : pos;
     const int per = (te - t0) * lpr;
     for (int i = threadIdx.x; i < 2 * per; i += kConsumerThreads) {
@@ -414,12 +493,15 @@ __device__ inline void att_prefetch_l2(const DecodeArgs& a, int l, int pos) {
 // Attention partials of this CTA's items for layer l at position pos. Item
 // (h, c): query head h over the positions of chunk c; publishes the chunk's
 // max score m, sum of exp(s - m), and sum of exp(s - m) * v.
+// With kB sequences the items are (sequence, head, chunk); sequence b has
+// its own q/k/v words, K/V cache, records and output.
+template <int kB>
 __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsigned tag_qkv,
                                        unsigned tag_att, float* sm, float* red, const Poll& pc) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int hd = a.hd, hd4 = hd >> 2, half = hd >> 1;
   int nch, clen;
-  att_split(pos, a.H, a.G, &nch, &clen);
+  att_split(pos, a.H * kB, a.G, &nch, &clen);
   const int group = a.H / a.Hkv;
   float* q = sm;             // hd
   float* kp = q + hd;        // hd: key of this position (after RoPE)
@@ -427,7 +509,6 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
   float* sc = vp + hd;       // clen <= kAttMaxChunk scores
   float* part = sc + kAttMaxChunk;  // 4 * kConsumerThreads
   const float2* rp = a.rope + (size_t)pos * half;
-  const size_t lay = (size_t)l * a.S * a.kvd;
   // lanes per position for the score dot products
   int lpp = 1;
   while (lpp < hd4 && lpp < 32) lpp <<= 1;
@@ -435,10 +516,14 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
   const int sub = lane / lpp, li = lane - sub * lpp;
 
   for (int pass = 0; pass < 2; ++pass)
-  for (int it = blockIdx.x; it < a.H * nch; it += a.G) {
-    const int h = it / nch, c = it - h * nch;
+  for (int it = blockIdx.x; it < kB * a.H * nch; it += a.G) {
+    const int b = kB == 1 ? 0 : it / (a.H * nch), hc = it - b * a.H * nch;
+    const int h = hc / nch, c = hc - h * nch;
     if ((c == 0) != (pass == 1)) continue;
     const int kvh = h / group;
+    const size_t lay = (size_t)b * a.kv_seq + (size_t)l * a.S * a.kvd;
+    const unsigned long long* xq = a.x_qkv + (size_t)b * (a.d + 2 * a.kvd);
+    const int hb = b * a.H + h;  // record and output index of (sequence, head)
     const int t0 = c * clen;
     const int t1 = (t0 + clen < pos + 1) ? t0 + clen : pos + 1;
     const bool has_new = (t1 == pos + 1);
@@ -468,7 +553,7 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
     for (int t = tid; t < nget && ok; t += kConsumerThreads) {
       const int which = t / half, i = t - which * half;
       const unsigned long long* src =
-          a.x_qkv + (which == 0 ? h * hd : a.d + (which - 1) * a.kvd + kvh * hd) + 2 * i;
+          xq + (which == 0 ? h * hd : a.d + (which - 1) * a.kvd + kvh * hd) + 2 * i;
       ulonglong2 v;
       ok = poll_one(src, tag_qkv, pc, v);
       const float x0 = lo_f(v.x), x1 = lo_f(v.y);
@@ -558,7 +643,7 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
     if (tid < hd)
       for (int g2 = 0; g2 < ng; ++g2) own += part[g2 * hd + tid];
     if (c != 0) {
-      unsigned long long* rec = a.x_att + ((size_t)h * a.nch_cap + c) * a.att_stride;
+      unsigned long long* rec = a.x_att + ((size_t)hb * a.nch_cap + c) * a.att_stride;
       if (tid < hd) st_tag(rec + 4 + tid, tag_att, own);
       if (tid == 0) {
         st_tag(rec, tag_att, m);
@@ -573,7 +658,7 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
           (nch - 1) * ppr,
           [&](int p) {
             const int cc = 1 + p / ppr, k = p - (cc - 1) * ppr;
-            const unsigned long long* r0 = a.x_att + ((size_t)h * a.nch_cap + cc) * a.att_stride;
+            const unsigned long long* r0 = a.x_att + ((size_t)hb * a.nch_cap + cc) * a.att_stride;
             return k == 0 ? r0 : r0 + 4 + 2 * (k - 1);
           },
           tag_att, pc, [&](int p, float x0, float x1) {
@@ -592,7 +677,7 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
         float o = (expf(m - M) / Lsum) * own;
         for (int cc = 0; cc < nch - 1; ++cc)
           o = fmaf(expf(mrg[cc * (hd + 2)] - M) / Lsum, mrg[cc * (hd + 2) + 2 + tid], o);
-        st_tag(a.x_attn + h * hd + tid, tag_att, o);
+        st_tag(a.x_attn + (size_t)hb * hd + tid, tag_att, o);
       }
     }
     named_bar_sync(kBarConsumers, kConsumerThreads);
@@ -600,19 +685,29 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
   return true;
 }
 
-// Next token: argmax over the per-CTA candidates (identical in every CTA).
+// Next token of each sequence: argmax over the per-CTA candidates
+// ([kB][G] pairs; identical in every CTA).
+template <int kB>
 __device__ inline bool reduce_candidates(const DecodeArgs& a, int parity, unsigned tag,
-                                         float* redv, int* redi, const Poll& pc, int* token) {
-  float bv = -INFINITY;
-  int bi = 0x7fffffff;
-  const unsigned long long* base = a.x_cand + (size_t)parity * a.G * 2;
-  const bool ok = poll_pairs(base, a.G, tag, pc, [&](int p, float v, float idx) {
-    const int i = (int)__float_as_uint(idx);
-    if (better(v, i, bv, bi)) { bv = v; bi = i; }
+                                         float* redv, int* redi, const Poll& pc,
+                                         int (&token)[kB]) {
+  float bv[kB];
+  int bi[kB];
+#pragma unroll
+  for (int b = 0; b < kB; ++b) { bv[b] = -INFINITY; bi[b] = 0x7fffffff; }
+  const unsigned long long* base = a.x_cand + (size_t)parity * kB * a.G * 2;
+  const bool ok = poll_pairs(base, kB * a.G, tag, pc, [&](int p, float v, float idx) {
+    const int i = (int)__float_as_uint(idx), pb = kB == 1 ? 0 : p / a.G;
+#pragma unroll
+    for (int b = 0; b < kB; ++b)
+      if (b == pb && better(v, i, bv[b], bi[b])) { bv[b] = v; bi[b] = i; }
   });
   if (!vote_ok(ok, pc.s_abort)) return false;
-  block_argmax(bv, bi, redv, redi);
-  *token = (bi >= 0 && bi < a.V) ? bi : 0;  // 0 only if every logit was NaN
+#pragma unroll
+  for (int b = 0; b < kB; ++b) {
+    block_argmax(bv[b], bi[b], redv, redi);
+    token[b] = (bi[b] >= 0 && bi[b] < a.V) ? bi[b] : 0;  // 0 only if every logit was NaN
+  }
   return true;
 }
 
@@ -660,7 +755,10 @@ struct DecodeSched {
   }
 };
 
-template <bool kQ8>
+// kB sequences decode in lockstep: sequence b's residual at xs + b d, its
+// phase input at vec + b vs, its words in every exchange buffer one vector
+// length after sequence b - 1's. The weights stream once for all of them.
+template <bool kQ8, int kB>
 __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned char* smem,
                                     volatile int* s_abort) {
   float* xs = reinterpret_cast<float*>(smem + a.sm_xs);
@@ -668,20 +766,26 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
   float* seg = reinterpret_cast<float*>(smem + a.sm_seg);
   float* asm_ = reinterpret_cast<float*>(smem + a.sm_att);
   float* red = reinterpret_cast<float*>(smem + a.sm_misc) + 8;
-  int* redi = reinterpret_cast<int*>(smem + a.sm_misc) + 24;
+  int* redi = reinterpret_cast<int*>(smem + a.sm_misc) + 80;
   const int tid = threadIdx.x, c = blockIdx.x;
+  const int vs = kB == 1 ? 0 : a.vs;
   const Poll pc{a.err, a.err_host, s_abort, a.wait_limit_ns};
   const unsigned per_step = (unsigned)(kPhasesPerLayer * a.L + 1);
   uint32_t g = 0;
-  int token = a.start_token;
-  // x += (published vector), identically in every CTA; ss += the new x^2
-  auto add_published = [&](const unsigned long long* src, unsigned tag, float& ss) {
-    const bool ok = poll_pairs(src, a.d >> 1, tag, pc, [&](int p, float v0, float v1) {
+  int token[kB];
+#pragma unroll
+  for (int b = 0; b < kB; ++b) token[b] = a.start_tokens[b];
+  // x += (published vector), identically in every CTA; ss[b] += the new x_b^2
+  auto add_published = [&](const unsigned long long* src, unsigned tag, float(&ss)[kB]) {
+    const int hp = a.d >> 1;
+    const bool ok = poll_pairs(src, kB * hp, tag, pc, [&](int p, float v0, float v1) {
       const float x0 = xs[2 * p] + v0, x1 = xs[2 * p + 1] + v1;
       xs[2 * p] = x0;
       xs[2 * p + 1] = x1;
-      ss = fmaf(x0, x0, ss);
-      ss = fmaf(x1, x1, ss);
+      const int pb = kB == 1 ? 0 : p / hp;
+#pragma unroll
+      for (int b = 0; b < kB; ++b)
+        if (b == pb) ss[b] = fmaf(x1, x1, fmaf(x0, x0, ss[b]));
     });
     return vote_ok(ok, s_abort);
   };
@@ -689,9 +793,10 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
     const int pos = a.start_pos + s;
     const unsigned es = a.epoch0 + (unsigned)s * per_step;
     if (s > 0) {
-      if (!reduce_candidates(a, (s - 1) & 1, es - 1, red, redi, pc, &token)) return false;
+      if (!reduce_candidates<kB>(a, (s - 1) & 1, es - 1, red, redi, pc, token)) return false;
       if (c == 0 && tid == 0) {
-        a.tokens[s - 1] = token;
+#pragma unroll
+        for (int b = 0; b < kB; ++b) a.tokens[(size_t)(s - 1) * kB + b] = token[b];
         a.ts[s - 1] = globaltimer_ns();
       }
     }
@@ -700,21 +805,25 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
     // barrier below order every later row load of the CTA after them.
     if (tid == 0) __threadfence();
     // x = E[token] (paper §4.1: weights are rows at offsets in the blob)
-    if (kQ8) {  // the row the codes stand for: scale * code
-      const unsigned char* er = a.q_E + (size_t)token * (16 + a.d);
-      const float sc = __ldg(reinterpret_cast<const float*>(er));
-      const int* cw = reinterpret_cast<const int*>(er + 16);
-      for (int j = tid; j < (a.d >> 2); j += kConsumerThreads) {
-        const int w = __ldg(cw + j);
-        reinterpret_cast<float4*>(xs)[j] =
-            make_float4(sc * (float)(int)(signed char)(w & 0xff),
-                        sc * (float)(int)(signed char)((w >> 8) & 0xff),
-                        sc * (float)(int)(signed char)((w >> 16) & 0xff), sc * (float)(w >> 24));
+#pragma unroll
+    for (int b = 0; b < kB; ++b) {
+      float* xb = xs + (size_t)b * a.d;
+      if (kQ8) {  // the row the codes stand for: scale * code
+        const unsigned char* er = a.q_E + (size_t)token[b] * (16 + a.d);
+        const float sc = __ldg(reinterpret_cast<const float*>(er));
+        const int* cw = reinterpret_cast<const int*>(er + 16);
+        for (int j = tid; j < (a.d >> 2); j += kConsumerThreads) {
+          const int w = __ldg(cw + j);
+          reinterpret_cast<float4*>(xb)[j] =
+              make_float4(sc * (float)(int)(signed char)(w & 0xff),
+                          sc * (float)(int)(signed char)((w >> 8) & 0xff),
+                          sc * (float)(int)(signed char)((w >> 16) & 0xff), sc * (float)(w >> 24));
+        }
+      } else {
+        const float4* e4 = reinterpret_cast<const float4*>(a.E + (size_t)token[b] * a.d);
+        for (int j = tid; j < (a.d >> 2); j += kConsumerThreads)
+          reinterpret_cast<float4*>(xb)[j] = __ldg(e4 + j);
       }
-    } else {
-      const float4* e4 = reinterpret_cast<const float4*>(a.E + (size_t)token * a.d);
-      for (int j = tid; j < (a.d >> 2); j += kConsumerThreads)
-        reinterpret_cast<float4*>(xs)[j] = __ldg(e4 + j);
     }
     named_bar_sync(kBarConsumers, kConsumerThreads);
     // The four GEMV phases of a layer run one copy of the phase code, in a
@@ -725,32 +834,46 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
       const unsigned el = es + (unsigned)(kPhasesPerLayer * l);
 #pragma unroll 1
       for (int k = 0; k < 4; ++k) {
-        if (k == 0) att_prefetch_l2(a, l, pos);
+        if (k == 0) att_prefetch_l2<kB>(a, l, pos);
         if (k == 0 || k == 2) {
           // x += (the previous phase's published output), then x_b = RMSNorm(x, g)
           const float* gain = reinterpret_cast<const float*>(lw + (k == 0 ? a.o_gatt : a.o_gffn));
           Gains gp;
           gp.load(gain, a.d);
-          float ss = 0.f;
+          float ss[kB];
+#pragma unroll
+          for (int b = 0; b < kB; ++b) ss[b] = 0.f;
           if (k == 2 || l > 0) {
             if (!add_published(k == 0 ? a.x_f : a.x_o, k == 0 ? el - 1 : el + 2, ss)) return false;
           } else {
-            ss = sum_sq(xs, a.d);
+#pragma unroll
+            for (int b = 0; b < kB; ++b) ss[b] = sum_sq(xs + (size_t)b * a.d, a.d);
           }
-          rmsnorm_finish(vec, xs, gp, gain, a.d, a.eps, ss, red);
+          rmsnorm_finish_n<kB>(vec, vs, xs, gp, gain, a.d, a.eps, ss, red);
         } else if (k == 1) {
-          if (!attention_phase(a, l, pos, el, el + 1, asm_, red, pc)) return false;
-          const bool ok = poll_pairs(a.x_attn, a.d >> 1, el + 1, pc, [&](int p, float v0, float v1) {
-            vec[2 * p] = v0;
-            vec[2 * p + 1] = v1;
+          if (!attention_phase<kB>(a, l, pos, el, el + 1, asm_, red, pc)) return false;
+          const int hp = a.d >> 1;
+          const bool ok = poll_pairs(a.x_attn, kB * hp, el + 1, pc, [&](int p, float v0, float v1) {
+            const int pb = kB == 1 ? 0 : p / hp;
+            float* dst = vec + (size_t)pb * vs + 2 * (p - pb * hp);
+            dst[0] = v0;
+            dst[1] = v1;
           });
           if (!vote_ok(ok, s_abort)) return false;
         } else {  // h = silu(a) * b (paper §2.1, SwiGLU); a = h13[i], b = h13[F + i]
-          const bool ok = poll_pairs2(a.x_h13, a.x_h13 + a.F, a.F >> 1, el + 3, pc,
-                                      [&](int p, float a0, float a1, float b0, float b1) {
-                                        vec[2 * p] = (a0 / (1.0f + expf(-a0))) * b0;
-                                        vec[2 * p + 1] = (a1 / (1.0f + expf(-a1))) * b1;
-                                      });
+          const int hp = a.F >> 1;
+          const bool ok = poll_pairs2(
+              kB * hp,
+              [&](int p) {
+                const int pb = kB == 1 ? 0 : p / hp;
+                return a.x_h13 + (size_t)pb * 2 * a.F + 2 * (p - pb * hp);
+              },
+              a.F, el + 3, pc, [&](int p, float a0, float a1, float b0, float b1) {
+                const int pb = kB == 1 ? 0 : p / hp;
+                float* dst = vec + (size_t)pb * vs + 2 * (p - pb * hp);
+                dst[0] = (a0 / (1.0f + expf(-a0))) * b0;
+                dst[1] = (a1 / (1.0f + expf(-a1))) * b1;
+              });
           if (!vote_ok(ok, s_abort)) return false;
         }
         // [Wq|Wk|Wv] x_b, Wo o, [W1|W3] x_b, W2 h: M rows of K columns, published
@@ -758,50 +881,70 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
         const int M = k == 0 ? a.d + 2 * a.kvd : k == 2 ? 2 * a.F : a.d;
         const int K = k == 3 ? a.F : a.d;
         unsigned long long* out = k == 0 ? a.x_qkv : k == 1 ? a.x_o : k == 2 ? a.x_h13 : a.x_f;
-        EpiTag e{out, el + (k == 0 ? 0u : (unsigned)k + 1u)};
-        if (!consume_phase<false, kQ8>(r, g, plan_stages(M, kQ8 ? 4 + K / 4 : K, a.G, c), vec, 1,
-                                       K, seg, e, a.err, a.err_host, s_abort))
-          return false;
+        EpiTag e{out, el + (k == 0 ? 0u : (unsigned)k + 1u), M};
+        if constexpr (kB == 1) {
+          if (!consume_phase<false, kQ8>(r, g, plan_stages(M, kQ8 ? 4 + K / 4 : K, a.G, c), vec,
+                                         1, K, seg, e, a.err, a.err_host, s_abort))
+            return false;
+        } else {
+          if (!consume_phase_b<kB>(r, g, plan_stages(M, K, a.G, c), vec, vs, seg, e, a.err,
+                                   a.err_host, s_abort))
+            return false;
+        }
       }
     }
     {
       Gains gp;
       gp.load(a.g_final, a.d);
-      float ss = 0.f;
+      float ss[kB];
+#pragma unroll
+      for (int b = 0; b < kB; ++b) ss[b] = 0.f;
       if (a.L > 0) {
         if (!add_published(a.x_f, es + per_step - 2, ss)) return false;
       } else {
-        ss = sum_sq(xs, a.d);
+#pragma unroll
+        for (int b = 0; b < kB; ++b) ss[b] = sum_sq(xs + (size_t)b * a.d, a.d);
       }
-      rmsnorm_finish(vec, xs, gp, a.g_final, a.d, a.eps, ss, red);
+      rmsnorm_finish_n<kB>(vec, vs, xs, gp, a.g_final, a.d, a.eps, ss, red);
     }
-    EpiArgmax ea{a.logits, -INFINITY, 0x7fffffff};
-    if (!consume_phase<false, kQ8>(r, g, plan_stages(a.V, kQ8 ? 4 + a.d / 4 : a.d, a.G, c), vec,
-                                   1, a.d, seg, ea, a.err, a.err_host, s_abort))
-      return false;
-    float bv = ea.bv;
-    int bi = ea.bi;
-    block_argmax(bv, bi, red, redi);
-    if (tid == 0) {
-      unsigned long long* dst = a.x_cand + ((size_t)(s & 1) * a.G + c) * 2;
-      st_tag(dst, es + per_step - 1, bv);
-      st_tag(dst + 1, es + per_step - 1, __uint_as_float((unsigned)bi));
+    EpiArgmax<kB> ea{a.logits, a.V};
+    ea.init();
+    if constexpr (kB == 1) {
+      if (!consume_phase<false, kQ8>(r, g, plan_stages(a.V, kQ8 ? 4 + a.d / 4 : a.d, a.G, c),
+                                     vec, 1, a.d, seg, ea, a.err, a.err_host, s_abort))
+        return false;
+    } else {
+      if (!consume_phase_b<kB>(r, g, plan_stages(a.V, a.d, a.G, c), vec, vs, seg, ea, a.err,
+                               a.err_host, s_abort))
+        return false;
+    }
+#pragma unroll
+    for (int b = 0; b < kB; ++b) {
+      float bv = ea.bv[b];
+      int bi = ea.bi[b];
+      block_argmax(bv, bi, red, redi);
+      if (tid == 0) {
+        unsigned long long* dst = a.x_cand + (((size_t)(s & 1) * kB + b) * a.G + c) * 2;
+        st_tag(dst, es + per_step - 1, bv);
+        st_tag(dst + 1, es + per_step - 1, __uint_as_float((unsigned)bi));
+      }
     }
   }
   if (a.final_token && c == 0) {
     const int s = a.n_steps - 1;
-    if (!reduce_candidates(a, s & 1, a.epoch0 + (unsigned)a.n_steps * per_step - 1, red, redi,
-                           pc, &token))
+    if (!reduce_candidates<kB>(a, s & 1, a.epoch0 + (unsigned)a.n_steps * per_step - 1, red,
+                               redi, pc, token))
       return false;
     if (tid == 0) {
-      a.tokens[s] = token;
+#pragma unroll
+      for (int b = 0; b < kB; ++b) a.tokens[(size_t)s * kB + b] = token[b];
       a.ts[s] = globaltimer_ns();
     }
   }
   return true;
 }
 
-template <bool kQ8>
+template <bool kQ8, int kB>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_constant__ DecodeArgs a) {
   extern __shared__ __align__(128) unsigned char smem[];
   Ring r;
@@ -829,20 +972,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
     }
     return;
   }
-  decode_steps<kQ8>(a, r, smem, s_abort);
+  decode_steps<kQ8, kB>(a, r, smem, s_abort);
 }
 
-// Failure-detection self-test: one CTA polls a tagged word that nothing
-// writes; the bounded wait must expire and report TVL_E_TIMEOUT.
-__global__ void wait_selftest_kernel(unsigned long long* word, int* err,
-                                     unsigned long long limit_ns) {
-  __shared__ int s_abort;
-  if (threadIdx.x == 0) s_abort = 0;
-  __syncthreads();
-  if (threadIdx.x >= kConsumerThreads) return;  // the consumer warps take part
-  const Poll pc{err, nullptr, &s_abort, limit_ns};
-  const bool ok = poll_pairs(word, 1, 1u, pc, [](int, float, float) {});
-  vote_ok(ok, &s_abort);
-}
+// decode_kernel<false, B> for B = 2..kMaxBatch (defined in decode_batch.cu).
+const void* decode_kernel_for_batch(int B);
 
 }  // namespace tvl

@@ -506,6 +506,146 @@ __device__ inline bool consume_phase(const Ring& r, uint32_t& g, const StagePlan
   return true;
 }
 
+// ---- several input vectors (batched decode) ----------------------------------------
+
+__host__ __device__ constexpr int pow2_at_least(int n) { return n <= 1 ? 1 : 2 * pow2_at_least((n + 1) / 2); }
+
+// Sums N values (N a power of two, at most 32) over the warp at once: after
+// the call lane l holds the warp's sum of v[l / (32 / N)]. Each halving step
+// trades half of a lane's values with its partner, so the warp spends N - 1 +
+// log2(32 / N) shuffles instead of 5 N.
+template <int N>
+__device__ __forceinline__ float warp_sum_transposed(float (&v)[N], int lane) {
+#pragma unroll
+  for (int t = 0; t < 5; ++t) {
+    const int o = 16 >> t;
+    const int cnt = (N >> t) > 1 ? (N >> t) : 1;
+    if (cnt > 1) {
+      const int half = cnt / 2;
+      const bool up = (lane & o) != 0;
+#pragma unroll
+      for (int i = 0; i < half; ++i) {
+        const float send = up ? v[i] : v[i + half];
+        const float keep = up ? v[i + half] : v[i];
+        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+      }
+    } else {
+      v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
+    }
+  }
+  return v[0];
+}
+
+// R rows of a stage (row r at w + r * ncols, ncols floats) times kB vectors
+// (vector b at x + b * vs): every weight float4 read from shared memory meets
+// all kB vectors, every x float4 all R rows. put(r, b, value) is called by
+// the lane that holds the sum of row r with vector b.
+template <int R, int kB, class Put>
+__device__ __forceinline__ void rows_times_vectors(const float* w, int ncols, const float* x,
+                                                   int vs, int lane, Put put) {
+  const int n4 = ncols >> 2, vs4 = vs >> 2;
+  const float4* w4 = reinterpret_cast<const float4*>(w);
+  const float4* x4 = reinterpret_cast<const float4*>(x);
+  // Few products: a float4 of partial sums each (four independent chains);
+  // many: one sum each (enough chains already, and fewer registers).
+  constexpr bool kWide = R * kB < 8;
+  constexpr int A = kWide ? 4 : 1;
+  float acc[R * kB][A];
+#pragma unroll
+  for (int i = 0; i < R * kB; ++i)
+#pragma unroll
+    for (int k = 0; k < A; ++k) acc[i][k] = 0.f;
+#pragma unroll 2
+  for (int e = lane; e < n4; e += 32) {
+    float4 wv[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) wv[r] = w4[r * n4 + e];
+#pragma unroll
+    for (int b = 0; b < kB; ++b) {
+      const float4 xv = x4[b * vs4 + e];
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        float* a = acc[r * kB + b];
+        if (kWide) {
+          a[0] = fmaf(wv[r].x, xv.x, a[0]);
+          a[A > 1 ? 1 : 0] = fmaf(wv[r].y, xv.y, a[A > 1 ? 1 : 0]);
+          a[A > 2 ? 2 : 0] = fmaf(wv[r].z, xv.z, a[A > 2 ? 2 : 0]);
+          a[A > 3 ? 3 : 0] = fmaf(wv[r].w, xv.w, a[A > 3 ? 3 : 0]);
+        } else {
+          a[0] = fmaf(wv[r].w, xv.w, fmaf(wv[r].z, xv.z, fmaf(wv[r].y, xv.y, fmaf(wv[r].x, xv.x, a[0]))));
+        }
+      }
+    }
+  }
+  constexpr int N = pow2_at_least(R * kB);
+  float v[N];
+#pragma unroll
+  for (int i = 0; i < N; ++i)
+    v[i] = i >= R * kB ? 0.f : kWide ? (acc[i][0] + acc[i][A > 1 ? 1 : 0]) + (acc[i][A > 2 ? 2 : 0] + acc[i][A > 3 ? 3 : 0]) : acc[i][0];
+  const float t = warp_sum_transposed<N>(v, lane);
+  const int idx = lane / (32 / N);
+  if (lane % (32 / N) == 0 && idx < R * kB) put(idx / kB, idx % kB, t);
+}
+
+// consume_phase for kB input vectors at once (vector b at xs + b * vs): the
+// same stages, each weight read once from the ring for all kB products.
+// epi.store_b(row, b, value) receives row `row` times vector b. Rows longer
+// than a stage leave kB partials per segment in seg, added in segment order.
+template <int kB, class Epi>
+__device__ inline bool consume_phase_b(const Ring& r, uint32_t& g, const StagePlan& p,
+                                       const float* xs, int vs, float* seg, Epi& epi, int* err,
+                                       int* err_host, volatile int* s_abort) {
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  bool ok = true;
+  int j = (int)((warp + kConsumerWarps - (int)(g % kConsumerWarps)) % kConsumerWarps);
+  for (; j < p.nstages && ok; j += kConsumerWarps) {
+    const uint32_t gs = g + (uint32_t)j;
+    const int slot = (int)(gs % (uint32_t)r.nst);
+    if (!warp_wait_full(r, slot, gs, err, err_host, s_abort)) {
+      ok = false;
+      break;
+    }
+    const StageDesc s = stage_desc(p, j);
+    const int ncols = s.c1 - s.c0;
+    const float* st = reinterpret_cast<const float*>(r.buf + (size_t)slot * kStageBytes);
+    const float* xb = xs + s.c0;
+    const int part = j % p.spr;
+    int ri = 0;
+    auto put_at = [&](int r0) {
+      return [&, r0](int rr, int b, float v) {
+        const int row = s.row + r0 + rr;
+        if (p.spr > 1) seg[((row - p.r0) * p.spr + part) * kB + b] = v;
+        else epi.store_b(row, b, v);
+      };
+    };
+    for (; ri + 4 <= s.nrows; ri += 4)
+      rows_times_vectors<4, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, put_at(ri));
+    if (ri + 2 <= s.nrows) {
+      rows_times_vectors<2, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, put_at(ri));
+      ri += 2;
+    }
+    if (ri < s.nrows)
+      rows_times_vectors<1, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, put_at(ri));
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&r.empty[slot]);  // stage free for the producer
+  }
+  g += (uint32_t)p.nstages;
+  if (named_bar_or(kBarConsumers, kConsumerThreads, !ok)) {
+    if (tid == 0) *s_abort = 1;
+    return false;
+  }
+  if (p.spr > 1) {  // rows longer than a stage: add the segments in order
+    for (int q = tid; q < (p.r1 - p.r0) * kB; q += kConsumerThreads) {
+      const int ri = q / kB, b = q - ri * kB;
+      float v = 0.f;
+      for (int k = 0; k < p.spr; ++k) v += seg[(ri * p.spr + k) * kB + b];
+      epi.store_b(p.r0 + ri, b, v);
+    }
+    named_bar_sync(kBarConsumers, kConsumerThreads);
+  }
+  return true;
+}
+
 struct EpiStore {
   float* out;
   __device__ __forceinline__ void store(int row, float v) { out[row] = v; }

@@ -32,6 +32,7 @@ class Config(ctypes.Structure):
         ("vocab_size", ctypes.c_int32), ("max_seq", ctypes.c_int32),
         ("rope_theta", ctypes.c_double), ("norm_eps", ctypes.c_double),
         ("shared_classifier", ctypes.c_int32), ("weight_bits", ctypes.c_int32),
+        ("max_batch", ctypes.c_int32),
     ]
 
 
@@ -42,6 +43,7 @@ class ModelInfo(ctypes.Structure):
         ("threads", ctypes.c_int32), ("smem_bytes", ctypes.c_int32),
         ("ring_stages", ctypes.c_int32), ("stage_bytes", ctypes.c_int32),
         ("tied", ctypes.c_int32), ("barriers_per_step", ctypes.c_int32),
+        ("max_batch", ctypes.c_int32),
     ]
 
 
@@ -62,6 +64,10 @@ def _load():
     L.tvl_forward.argtypes = [P, i32, i32, P]
     L.tvl_decode_greedy.restype = st
     L.tvl_decode_greedy.argtypes = [P, i32, i32, i32, P]
+    L.tvl_forward_batch.restype = st
+    L.tvl_forward_batch.argtypes = [P, i32, P, i32, P]
+    L.tvl_decode_greedy_batch.restype = st
+    L.tvl_decode_greedy_batch.argtypes = [P, i32, P, i32, i32, P]
     L.tvl_gemv.restype = st
     L.tvl_gemv.argtypes = [P, P, P, i32, i32, P]
     L.tvl_q8_bytes.restype = sz
@@ -92,6 +98,7 @@ def _load():
 lib = _load()
 
 EXPORTED = ["tvl_blob_bytes", "tvl_load", "tvl_load_file", "tvl_forward", "tvl_decode_greedy",
+            "tvl_forward_batch", "tvl_decode_greedy_batch",
             "tvl_gemv", "tvl_gemv_noalloc", "tvl_q8_bytes", "tvl_quantize_q8", "tvl_gemv_q8",
             "tvl_sync", "tvl_free", "tvl_status_string", "tvl_last_error",
             "tvl_get_info", "tvl_step_times", "tvl_selftest_barrier_timeout"]
@@ -116,6 +123,7 @@ def make_config(cfg: dict) -> Config:
         int(cfg["n_kv_heads"]), int(cfg["vocab_size"]), int(cfg["max_seq"]),
         float(cfg.get("rope_theta", 10000.0)), float(cfg.get("norm_eps", 1e-5)),
         int(cfg.get("shared_classifier", 0)), int(cfg.get("weight_bits", 0)),
+        int(cfg.get("max_batch", 0)),
     )
 
 
@@ -212,6 +220,32 @@ class Model:
         ptr = ctypes.c_void_p(out.ctypes.data) if tokens else None
         _check(lib.tvl_decode_greedy(self._h, int(start_token), int(start_pos), int(n_steps),
                                      ptr), "tvl_decode_greedy")
+        return out
+
+    def forward_batch(self, tokens, pos: int, logits=None):
+        """One step of len(tokens) sequences at position pos. logits: None,
+        a float32 numpy array of batch * V (host: the call waits), or an
+        integer device address (async); laid out [batch][V]."""
+        toks = np.ascontiguousarray(tokens, dtype=np.int32)
+        if logits is None:
+            ptr = None
+        else:
+            if isinstance(logits, np.ndarray):
+                assert logits.dtype == np.float32 and logits.size >= toks.size * self.vocab
+            ptr = ctypes.c_void_p(_addr(logits))
+        _check(lib.tvl_forward_batch(self._h, int(toks.size), ctypes.c_void_p(toks.ctypes.data),
+                                     int(pos), ptr), "tvl_forward_batch")
+        return logits
+
+    def decode_greedy_batch(self, start_tokens, start_pos: int, n_steps: int, tokens=True):
+        """Greedy decoding of len(start_tokens) sequences in lockstep; returns
+        int32 [n_steps, batch] (or None when tokens=False: no copy, no wait)."""
+        toks = np.ascontiguousarray(start_tokens, dtype=np.int32)
+        out = np.empty((int(n_steps), toks.size), dtype=np.int32) if tokens else None
+        ptr = ctypes.c_void_p(out.ctypes.data) if tokens else None
+        _check(lib.tvl_decode_greedy_batch(self._h, int(toks.size),
+                                           ctypes.c_void_p(toks.ctypes.data), int(start_pos),
+                                           int(n_steps), ptr), "tvl_decode_greedy_batch")
         return out
 
     def step_times(self, n: int) -> np.ndarray:

@@ -60,6 +60,9 @@ def test_blob_bytes_agree_with_generator_and_oracle(tvl):
     (dict(dim=256, n_heads=1, n_kv_heads=1), "E_UNSUPPORTED"),  # head_dim 256 > 128
     (dict(weight_bits=4), "E_INVAL"),                           # 0 or 8 only
     (dict(weight_bits=8, hidden_dim=104), "E_UNSUPPORTED"),     # 8-bit rows: 104 % 16 != 0
+    (dict(max_batch=5), "E_INVAL"),                             # 0 to 4 sequences
+    (dict(max_batch=-1), "E_INVAL"),
+    (dict(max_batch=2, weight_bits=8), "E_UNSUPPORTED"),        # batches need float32 rows
 ])
 def test_load_rejects_invalid_configs_on_the_host(tvl, bad, status):
     cfg = dict(dim=64, hidden_dim=96, n_layers=1, n_heads=4, n_kv_heads=4, vocab_size=100,
