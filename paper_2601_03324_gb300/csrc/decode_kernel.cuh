@@ -151,14 +151,14 @@ struct PollClock {
 // batch is re-read together, so waiting costs one round trip after the last
 // producer's store. fn(p, v0, v1) takes each ready pair. Returns false if this
 // thread gave up (the caller votes).
-template <class Fn>
+template <int D = 4, class Fn>
 __device__ inline bool poll_pairs(const unsigned long long* src, int npairs, unsigned tag,
                                   const Poll& c, Fn fn) {
-  for (int base = threadIdx.x; base < npairs; base += kConsumerThreads * 4) {
-    ulonglong2 v[4];
+  for (int base = threadIdx.x; base < npairs; base += kConsumerThreads * D) {
+    ulonglong2 v[D];
     unsigned pending = 0;
 #pragma unroll
-    for (int b = 0; b < 4; ++b) {
+    for (int b = 0; b < D; ++b) {
       const int p = base + b * kConsumerThreads;
       if (p < npairs) {
         v[b] = ld_tag2(src + 2 * p);
@@ -168,7 +168,7 @@ __device__ inline bool poll_pairs(const unsigned long long* src, int npairs, uns
     PollClock clk;
     while (true) {
 #pragma unroll
-      for (int b = 0; b < 4; ++b) {
+      for (int b = 0; b < D; ++b) {
         if ((pending >> b) & 1u) {
           if (tags_are(v[b], tag)) {
             fn(base + b * kConsumerThreads, lo_f(v[b].x), lo_f(v[b].y));
@@ -179,7 +179,7 @@ __device__ inline bool poll_pairs(const unsigned long long* src, int npairs, uns
       if (!pending) break;
       if (!clk.keep_waiting(c)) return false;
 #pragma unroll
-      for (int b = 0; b < 4; ++b)
+      for (int b = 0; b < D; ++b)
         if ((pending >> b) & 1u) v[b] = ld_tag2(src + 2 * (base + b * kConsumerThreads));
     }
   }
@@ -188,14 +188,14 @@ __device__ inline bool poll_pairs(const unsigned long long* src, int npairs, uns
 
 // Same, over two tagged vectors read in step: the pair at addr(p) and the
 // one `off` words after it; fn(p, a0, a1, b0, b1).
-template <class Addr, class Fn>
+template <int D = 4, class Addr, class Fn>
 __device__ inline bool poll_pairs2(int npairs, Addr addr, long long off, unsigned tag,
                                    const Poll& c, Fn fn) {
-  for (int base = threadIdx.x; base < npairs; base += kConsumerThreads * 4) {
-    ulonglong2 va[4], vb[4];
+  for (int base = threadIdx.x; base < npairs; base += kConsumerThreads * D) {
+    ulonglong2 va[D], vb[D];
     unsigned pending = 0;
 #pragma unroll
-    for (int b = 0; b < 4; ++b) {
+    for (int b = 0; b < D; ++b) {
       const int p = base + b * kConsumerThreads;
       if (p < npairs) {
         va[b] = ld_tag2(addr(p));
@@ -206,7 +206,7 @@ __device__ inline bool poll_pairs2(int npairs, Addr addr, long long off, unsigne
     PollClock clk;
     while (true) {
 #pragma unroll
-      for (int b = 0; b < 4; ++b) {
+      for (int b = 0; b < D; ++b) {
         if (((pending >> b) & 1u) && tags_are(va[b], tag) && tags_are(vb[b], tag)) {
           fn(base + b * kConsumerThreads, lo_f(va[b].x), lo_f(va[b].y), lo_f(vb[b].x),
              lo_f(vb[b].y));
@@ -216,7 +216,7 @@ __device__ inline bool poll_pairs2(int npairs, Addr addr, long long off, unsigne
       if (!pending) break;
       if (!clk.keep_waiting(c)) return false;
 #pragma unroll
-      for (int b = 0; b < 4; ++b) {
+      for (int b = 0; b < D; ++b) {
         if ((pending >> b) & 1u) {
           const int p = base + b * kConsumerThreads;
           va[b] = ld_tag2(addr(p));
@@ -769,6 +769,10 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
   int* redi = reinterpret_cast<int*>(smem + a.sm_misc) + 80;
   const int tid = threadIdx.x, c = blockIdx.x;
   const int vs = kB == 1 ? 0 : a.vs;
+  // 16-byte polls in flight per thread (two loads per pair for h13): one
+  // batch covers a 768-wide vector, and h13's 1024 pairs at hidden width 2048
+  constexpr int kPollDepth = 4;
+  constexpr int kPollDepthH = kB == 1 ? 5 : 4;
   const Poll pc{a.err, a.err_host, s_abort, a.wait_limit_ns};
   const unsigned per_step = (unsigned)(kPhasesPerLayer * a.L + 1);
   uint32_t g = 0;
@@ -778,7 +782,7 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
   // x += (published vector), identically in every CTA; ss[b] += the new x_b^2
   auto add_published = [&](const unsigned long long* src, unsigned tag, float(&ss)[kB]) {
     const int hp = a.d >> 1;
-    const bool ok = poll_pairs(src, kB * hp, tag, pc, [&](int p, float v0, float v1) {
+    const bool ok = poll_pairs<kPollDepth>(src, kB * hp, tag, pc, [&](int p, float v0, float v1) {
       const float x0 = xs[2 * p] + v0, x1 = xs[2 * p + 1] + v1;
       xs[2 * p] = x0;
       xs[2 * p + 1] = x1;
@@ -853,7 +857,8 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
         } else if (k == 1) {
           if (!attention_phase<kB>(a, l, pos, el, el + 1, asm_, red, pc)) return false;
           const int hp = a.d >> 1;
-          const bool ok = poll_pairs(a.x_attn, kB * hp, el + 1, pc, [&](int p, float v0, float v1) {
+          const bool ok = poll_pairs<kPollDepth>(a.x_attn, kB * hp, el + 1, pc,
+                                                 [&](int p, float v0, float v1) {
             const int pb = kB == 1 ? 0 : p / hp;
             float* dst = vec + (size_t)pb * vs + 2 * (p - pb * hp);
             dst[0] = v0;
@@ -862,7 +867,7 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
           if (!vote_ok(ok, s_abort)) return false;
         } else {  // h = silu(a) * b (paper §2.1, SwiGLU); a = h13[i], b = h13[F + i]
           const int hp = a.F >> 1;
-          const bool ok = poll_pairs2(
+          const bool ok = poll_pairs2<kPollDepthH>(
               kB * hp,
               [&](int p) {
                 const int pb = kB == 1 ? 0 : p / hp;
