@@ -134,6 +134,20 @@ bool is_device_pointer(const void* p) {
   return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
 }
 
+// Interleaves the rows of a [W1 | W3] block in place (F rows of row_bytes
+// each, then F more): row 2i becomes W1's row i and row 2i + 1 W3's, so that
+// one CTA computes both halves of each SwiGLU product. tmp holds the block.
+tvl_status interleave_w13(unsigned char* block, size_t F, size_t row_bytes, unsigned char* tmp,
+                          cudaStream_t st) {
+  const size_t half = F * row_bytes;
+  TVL_CK(cudaMemcpyAsync(tmp, block, 2 * half, cudaMemcpyDeviceToDevice, st));
+  TVL_CK(cudaMemcpy2DAsync(block, 2 * row_bytes, tmp, row_bytes, row_bytes, F,
+                           cudaMemcpyDeviceToDevice, st));
+  TVL_CK(cudaMemcpy2DAsync(block + row_bytes, 2 * row_bytes, tmp + half, row_bytes, row_bytes, F,
+                           cudaMemcpyDeviceToDevice, st));
+  return TVL_OK;
+}
+
 tvl_status launch(tvl_model* m, int B, const int* tokens, int pos, int n_steps,
                   int final_token) {
   DecodeArgs a = m->args;
@@ -240,8 +254,8 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
       const long long Ms[5] = {d + 2LL * kvd, d, 2LL * F, d, V};
       const int Ks[5] = {d, d, d, F, d};
       for (int i = 0; i < 5; ++i) {
-        const StagePlan pl = plan_stages(Ms[i], Ks[i], G, 0);
-        if (pl.spr > 1 && (long long)((Ms[i] + G - 1) / G) * pl.spr * B > kMaxSegParts) {
+        const StagePlan pl = plan_stages(Ms[i], Ks[i], G, 0, i == 2 ? 2 : 1);
+        if (pl.defer && (long long)((Ms[i] + G - 1) / G + 1) * pl.spr * B > kMaxSegParts) {
           set_error("tvl_load: too many long rows per SM for the segment scratch");
           return fail(TVL_E_UNSUPPORTED);
         }
@@ -308,7 +322,7 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   const size_t o_scr = off;
   const size_t nB = (size_t)maxB;
   const size_t o_qkv = take(8ull * (d + 2 * kvd) * nB), o_o = take(8ull * d * nB);
-  const size_t o_h13 = take(16ull * F * nB);
+  const size_t o_h13 = take(8ull * F * nB);
   const size_t o_f = take(8ull * d * nB), o_lg = take(4ull * V * nB);
   const size_t o_att = take(8ull * H * nch_cap * att_stride * nB);
   const size_t o_attn = take(8ull * d * nB);
@@ -378,6 +392,21 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
     if (st == TVL_OK) st = quant(Wf + bl.E, o_qE, V, d);
     if (st == TVL_OK && !tied) st = quant(Wf + bl.Wcls, o_qcls, V, d);
     if (st == TVL_OK) st = ck(cudaStreamSynchronize(m->stream), "cudaStreamSynchronize(q8)");
+    if (st != TVL_OK) return fail(st);
+  }
+  {  // the streamed [W1 | W3] blocks get interleaved rows
+    const size_t row_bytes = q8 ? rq : 4ull * d;
+    unsigned char* tmp = nullptr;
+    if (L > 0 && (st = ck(cudaMalloc((void**)&tmp, 2 * (size_t)F * row_bytes),
+                          "cudaMalloc(w13 scratch)")) != TVL_OK)
+      return fail(st);
+    for (int l = 0; l < L && st == TVL_OK; ++l) {
+      unsigned char* blk = q8 ? m->arena + o_q + (size_t)l * q_stride + q_w13
+                              : m->arena + o_w + bl.l0 + (size_t)l * bl.stride + bl.w1;
+      st = interleave_w13(blk, (size_t)F, row_bytes, tmp, m->stream);
+    }
+    if (st == TVL_OK) st = ck(cudaStreamSynchronize(m->stream), "cudaStreamSynchronize(w13)");
+    if (tmp) cudaFree(tmp);
     if (st != TVL_OK) return fail(st);
   }
 

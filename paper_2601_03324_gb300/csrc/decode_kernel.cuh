@@ -7,8 +7,11 @@
 //   2. RoPE on q, k; k, v into the cache; attention partials per
 //      (head, position chunk)                              (items split over CTAs)
 //   3. o = merge of the partials; y = Wo o
-//   4. x += y; x_b = RMSNorm(x, g_ffn); [a|b] = W13 x_b
-//   5. h = silu(a) * b; y = W2 h; then x += y
+//   4. x += y; x_b = RMSNorm(x, g_ffn); a = W1 x_b, b = W3 x_b, and
+//      h = silu(a) * b where a_i and b_i are computed (the device copy of
+//      W1 and W3 interleaves their rows: row 2i is W1's row i, row 2i + 1
+//      W3's)                                                (row pairs split over CTAs)
+//   5. y = W2 h; then x += y
 // and after the last layer: x_b = RMSNorm(x, g_final); logits = Wcls x_b with
 // a per-CTA argmax. The residual stream x is held, identically, in every
 // CTA's shared memory: each CTA adds the same values in the same order.
@@ -59,7 +62,7 @@ struct DecodeArgs {
   unsigned long long* x_att;   // [H][nch_cap][att_stride]: m, l, -, -, sum[hd] of chunks > 0
   unsigned long long* x_attn;  // [d]: attention output, merged per head
   unsigned long long* x_o;     // [d]
-  unsigned long long* x_h13;   // [2F]
+  unsigned long long* x_h13;   // [F]: h = silu(W1 x_b) * (W3 x_b)
   unsigned long long* x_f;     // [d]
   unsigned long long* x_cand;  // [2][G][2]: per step parity, per CTA (value, index)
   float* logits;               // [V]
@@ -181,48 +184,6 @@ __device__ inline bool poll_pairs(const unsigned long long* src, int npairs, uns
 #pragma unroll
       for (int b = 0; b < D; ++b)
         if ((pending >> b) & 1u) v[b] = ld_tag2(src + 2 * (base + b * kConsumerThreads));
-    }
-  }
-  return true;
-}
-
-// Same, over two tagged vectors read in step: the pair at addr(p) and the
-// one `off` words after it; fn(p, a0, a1, b0, b1).
-template <int D = 4, class Addr, class Fn>
-__device__ inline bool poll_pairs2(int npairs, Addr addr, long long off, unsigned tag,
-                                   const Poll& c, Fn fn) {
-  for (int base = threadIdx.x; base < npairs; base += kConsumerThreads * D) {
-    ulonglong2 va[D], vb[D];
-    unsigned pending = 0;
-#pragma unroll
-    for (int b = 0; b < D; ++b) {
-      const int p = base + b * kConsumerThreads;
-      if (p < npairs) {
-        va[b] = ld_tag2(addr(p));
-        vb[b] = ld_tag2(addr(p) + off);
-        pending |= 1u << b;
-      }
-    }
-    PollClock clk;
-    while (true) {
-#pragma unroll
-      for (int b = 0; b < D; ++b) {
-        if (((pending >> b) & 1u) && tags_are(va[b], tag) && tags_are(vb[b], tag)) {
-          fn(base + b * kConsumerThreads, lo_f(va[b].x), lo_f(va[b].y), lo_f(vb[b].x),
-             lo_f(vb[b].y));
-          pending &= ~(1u << b);
-        }
-      }
-      if (!pending) break;
-      if (!clk.keep_waiting(c)) return false;
-#pragma unroll
-      for (int b = 0; b < D; ++b) {
-        if ((pending >> b) & 1u) {
-          const int p = base + b * kConsumerThreads;
-          va[b] = ld_tag2(addr(p));
-          vb[b] = ld_tag2(addr(p) + off);
-        }
-      }
     }
   }
   return true;
@@ -432,13 +393,28 @@ __device__ inline float sum_sq(const float* x, int n) {
   return ss;
 }
 
+// Publishes GEMV rows as tagged words (M words per sequence). With swiglu
+// the rows are interleaved pairs (W1 row i, W3 row i) and the pair publishes
+// h_i = silu(a_i) * b_i at word i instead (paper §2.1, SwiGLU).
 struct EpiTag {
   unsigned long long* out;
   unsigned tag;
-  int M;  // words between two sequences' outputs
-  __device__ __forceinline__ void store(int row, float v) { st_tag(out + row, tag, v); }
+  int M;
+  bool swiglu;
+  __device__ __forceinline__ void store(int row, float v) { store_b(row, 0, v); }
   __device__ __forceinline__ void store_b(int row, int b, float v) {
     st_tag(out + (size_t)b * M + row, tag, v);
+  }
+  __device__ __forceinline__ void store_pair(int row, float v0, float v1) {
+    store_pair_b(row, 0, v0, v1);
+  }
+  __device__ __forceinline__ void store_pair_b(int row, int b, float v0, float v1) {
+    if (swiglu) {
+      st_tag(out + (size_t)b * M + (row >> 1), tag, (v0 / (1.0f + expf(-v0))) * v1);
+    } else {
+      st_tag(out + (size_t)b * M + row, tag, v0);
+      st_tag(out + (size_t)b * M + row + 1, tag, v1);
+    }
   }
 };
 
@@ -455,6 +431,14 @@ struct EpiArgmax {
     for (int b = 0; b < kB; ++b) { bv[b] = -INFINITY; bi[b] = 0x7fffffff; }
   }
   __device__ __forceinline__ void store(int row, float v) { store_b(row, 0, v); }
+  __device__ __forceinline__ void store_pair(int row, float v0, float v1) {
+    store_b(row, 0, v0);
+    store_b(row + 1, 0, v1);
+  }
+  __device__ __forceinline__ void store_pair_b(int row, int b, float v0, float v1) {
+    store_b(row, b, v0);
+    store_b(row + 1, b, v1);
+  }
   __device__ __forceinline__ void store_b(int row, int b, float v) {
     out[(size_t)b * V + row] = v;
 #pragma unroll
@@ -714,7 +698,8 @@ __device__ inline bool reduce_candidates(const DecodeArgs& a, int parity, unsign
 // ---- the kernel --------------------------------------------------------------------
 
 // The weight stream of one launch, in consumption order: per step, each
-// layer's [Wq|Wk|Wv], Wo, [W1|W3], W2, then the classifier; this CTA's rows.
+// layer's [Wq|Wk|Wv], Wo, W1/W3 (interleaved rows), W2, then the classifier;
+// this CTA's rows.
 template <bool kQ8>
 struct DecodeSched {
   const DecodeArgs* a;
@@ -735,7 +720,7 @@ struct DecodeSched {
         p = plan_stages(a->d, kQ8 ? 4 + a->d / 4 : a->d, a->G, c);
       } else if (k == 2) {
         W = reinterpret_cast<const float*>(kQ8 ? ql + a->q_w13 : lw + a->o_w13);
-        p = plan_stages(2 * a->F, kQ8 ? 4 + a->d / 4 : a->d, a->G, c);
+        p = plan_stages(2 * a->F, kQ8 ? 4 + a->d / 4 : a->d, a->G, c, 2);
       } else {
         W = reinterpret_cast<const float*>(kQ8 ? ql + a->q_w2 : lw + a->o_w2);
         p = plan_stages(a->d, kQ8 ? 4 + a->F / 4 : a->F, a->G, c);
@@ -769,10 +754,10 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
   int* redi = reinterpret_cast<int*>(smem + a.sm_misc) + 80;
   const int tid = threadIdx.x, c = blockIdx.x;
   const int vs = kB == 1 ? 0 : a.vs;
-  // 16-byte polls in flight per thread (two loads per pair for h13): one
-  // batch covers a 768-wide vector, and h13's 1024 pairs at hidden width 2048
+  // 16-byte polls in flight per thread: one batch covers a 768-wide vector,
+  // and the 1024 pairs of h at hidden width 2048
   constexpr int kPollDepth = 4;
-  constexpr int kPollDepthH = kB == 1 ? 5 : 4;
+  constexpr int kPollDepthH = kB == 1 ? 5 : 8;
   const Poll pc{a.err, a.err_host, s_abort, a.wait_limit_ns};
   const unsigned per_step = (unsigned)(kPhasesPerLayer * a.L + 1);
   uint32_t g = 0;
@@ -865,35 +850,31 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
             dst[1] = v1;
           });
           if (!vote_ok(ok, s_abort)) return false;
-        } else {  // h = silu(a) * b (paper §2.1, SwiGLU); a = h13[i], b = h13[F + i]
+        } else {  // h, published by the W1/W3 phase
           const int hp = a.F >> 1;
-          const bool ok = poll_pairs2<kPollDepthH>(
-              kB * hp,
-              [&](int p) {
-                const int pb = kB == 1 ? 0 : p / hp;
-                return a.x_h13 + (size_t)pb * 2 * a.F + 2 * (p - pb * hp);
-              },
-              a.F, el + 3, pc, [&](int p, float a0, float a1, float b0, float b1) {
-                const int pb = kB == 1 ? 0 : p / hp;
-                float* dst = vec + (size_t)pb * vs + 2 * (p - pb * hp);
-                dst[0] = (a0 / (1.0f + expf(-a0))) * b0;
-                dst[1] = (a1 / (1.0f + expf(-a1))) * b1;
-              });
+          const bool ok = poll_pairs<kPollDepthH>(a.x_h13, kB * hp, el + 3, pc,
+                                                  [&](int p, float v0, float v1) {
+            const int pb = kB == 1 ? 0 : p / hp;
+            float* dst = vec + (size_t)pb * vs + 2 * (p - pb * hp);
+            dst[0] = v0;
+            dst[1] = v1;
+          });
           if (!vote_ok(ok, s_abort)) return false;
         }
-        // [Wq|Wk|Wv] x_b, Wo o, [W1|W3] x_b, W2 h: M rows of K columns, published
-        // with the exchange tag of phase k (the attention partials take el + 1)
+        // [Wq|Wk|Wv] x_b, Wo o, W1/W3 x_b (row pairs: h), W2 h: M rows of K
+        // columns, published with the exchange tag of phase k (the attention
+        // partials take el + 1)
         const int M = k == 0 ? a.d + 2 * a.kvd : k == 2 ? 2 * a.F : a.d;
         const int K = k == 3 ? a.F : a.d;
+        const StagePlan plan = plan_stages(M, kQ8 ? 4 + K / 4 : K, a.G, c, k == 2 ? 2 : 1);
         unsigned long long* out = k == 0 ? a.x_qkv : k == 1 ? a.x_o : k == 2 ? a.x_h13 : a.x_f;
-        EpiTag e{out, el + (k == 0 ? 0u : (unsigned)k + 1u), M};
+        EpiTag e{out, el + (k == 0 ? 0u : (unsigned)k + 1u), k == 2 ? a.F : M, k == 2};
         if constexpr (kB == 1) {
-          if (!consume_phase<false, kQ8>(r, g, plan_stages(M, kQ8 ? 4 + K / 4 : K, a.G, c), vec,
-                                         1, K, seg, e, a.err, a.err_host, s_abort))
+          if (!consume_phase<false, kQ8>(r, g, plan, vec, 1, K, seg, e, a.err, a.err_host,
+                                         s_abort))
             return false;
         } else {
-          if (!consume_phase_b<kB>(r, g, plan_stages(M, K, a.G, c), vec, vs, seg, e, a.err,
-                                   a.err_host, s_abort))
+          if (!consume_phase_b<kB>(r, g, plan, vec, vs, seg, e, a.err, a.err_host, s_abort))
             return false;
         }
       }

@@ -36,6 +36,10 @@ struct GemvArgs {
 struct EpiPart {
   float* part;
   __device__ __forceinline__ void store(int v, float val) { part[v] = val; }
+  __device__ __forceinline__ void store_pair(int v, float v0, float v1) {
+    part[v] = v0;
+    part[v + 1] = v1;
+  }
 };
 
 // The single phase of a standalone GEMV.

@@ -51,6 +51,8 @@ struct StagePlan {
   int spr;  // stages per row when it does not (else 1)
   int seg;  // floats per segment when spr > 1 (multiple of 32)
   int nstages;
+  int gran;    // 2: rows come in pairs (2i, 2i+1) whose results meet in one epilogue call
+  bool defer;  // results wait in the segment scratch and are stored at the end of the phase
 };
 
 struct StageDesc {
@@ -58,12 +60,19 @@ struct StageDesc {
 };
 
 // Requires K % 4 == 0 (16-byte rows) and kStageFloats % 32 == 0. A stage has
-// at most kMaxRowsPerStage rows, or one segment of at most kStageFloats.
-__host__ __device__ inline StagePlan plan_stages(long long M, int K, int G, int c) {
+// at most kMaxRowsPerStage rows, or one segment of at most kStageFloats. With
+// gran 2 (M even) a CTA owns whole pairs of rows and a stage holds whole
+// pairs, unless a pair does not fit a stage: then the rows' results are
+// deferred to the end of the phase, like the segments of rows longer than a
+// stage.
+__host__ __device__ inline StagePlan plan_stages(long long M, int K, int G, int c,
+                                                 int gran = 1) {
   StagePlan p;
-  p.r0 = (int)(M * c / G);
-  p.r1 = (int)(M * (c + 1) / G);
+  p.gran = gran;
+  p.r0 = gran * (int)((M / gran) * c / G);
+  p.r1 = gran * (int)((M / gran) * (c + 1) / G);
   p.K = K;
+  p.defer = false;
   const int nrows = p.r1 - p.r0;
   if (K <= kStageFloats) {
     // rows per stage: as many as fit, but few enough that the CTA's rows of
@@ -73,7 +82,10 @@ __host__ __device__ inline StagePlan plan_stages(long long M, int K, int G, int 
     if (cap > kMaxRowsPerStage) cap = kMaxRowsPerStage;
     int spread = (nrows + kConsumerWarps - 1) / kConsumerWarps;
     if (spread < 1) spread = 1;
+    if (gran == 2) spread += spread & 1;
     p.rps = spread < cap ? spread : cap;
+    if (gran == 2 && p.rps >= 2) p.rps &= ~1;
+    p.defer = gran == 2 && p.rps < 2;
     p.spr = 1;
     p.seg = K;
     p.nstages = (nrows + p.rps - 1) / p.rps;
@@ -82,6 +94,7 @@ __host__ __device__ inline StagePlan plan_stages(long long M, int K, int G, int 
     p.spr = (K + kStageFloats - 1) / kStageFloats;
     p.seg = ((K + p.spr - 1) / p.spr + 31) / 32 * 32;
     p.nstages = nrows * p.spr;
+    p.defer = true;
   }
   return p;
 }
@@ -387,10 +400,11 @@ __device__ inline bool warp_wait_full(const Ring& r, int slot, uint32_t gs, int*
 // Consumer: one GEMV phase over the CTA's stage plan. The input vector xs is
 // in shared memory; with S > 1 the matrix is viewed as [M*S x Kc] "virtual
 // rows" (row r, K-chunk s) and virtual row v reads xs + (v % S) * Kc.
-// epi.store(v, value) receives each finished (virtual) row, from lane 0 of
-// the warp that computed it, or (rows longer than a stage) from the thread
-// that adds the row's segment partials at the end of the phase. seg is
-// shared scratch for those partials. Ends with a barrier of the consumer
+// epi.store(v, value) receives each finished (virtual) row, or
+// epi.store_pair(v, value_v, value_v+1) two rows v (even with gran 2) and
+// v + 1 computed together, from lane 0 of the warp that computed them, or
+// (deferred rows) from the thread that adds the rows' partials at the end of
+// the phase. seg is shared scratch for those partials. Ends with a barrier of the consumer
 // warps; returns false on abort, identically in every consumer thread.
 template <bool kXReg = true, bool kQ8 = false, class Epi>
 __device__ inline bool consume_phase(const Ring& r, uint32_t& g, const StagePlan& p,
@@ -443,8 +457,9 @@ __device__ inline bool consume_phase(const Ring& r, uint32_t& g, const StagePlan
           a1 += __shfl_xor_sync(0xffffffffu, a1, o);
         }
         if (lane == 0) {
-          epi.store(s.row + ri, r0[0] * a0);
-          if (two) epi.store(s.row + ri + 1, r1[0] * a1);
+          if (p.defer) seg[s.row + ri - p.r0] = r0[0] * a0;
+          else if (two) epi.store_pair(s.row + ri, r0[0] * a0, r1[0] * a1);
+          else epi.store(s.row + ri, r0[0] * a0);
         }
       }
       __syncwarp();
@@ -478,11 +493,12 @@ __device__ inline bool consume_phase(const Ring& r, uint32_t& g, const StagePlan
         a1 += __shfl_xor_sync(0xffffffffu, a1, o);
       }
       if (lane == 0) {
-        if (p.spr > 1) {
+        if (p.defer) {  // one row (or segment) per stage
           seg[(v0 - p.r0) * p.spr + j % p.spr] = a0;
+        } else if (two) {
+          epi.store_pair(v0, a0, a1);
         } else {
           epi.store(v0, a0);
-          if (two) epi.store(v1, a1);
         }
       }
     }
@@ -495,11 +511,16 @@ __device__ inline bool consume_phase(const Ring& r, uint32_t& g, const StagePlan
     if (tid == 0) *s_abort = 1;
     return false;
   }
-  if (p.spr > 1) {  // rows longer than a stage: add the segments in order
-    for (int ri = tid; ri < p.r1 - p.r0; ri += kConsumerThreads) {
+  if (p.defer) {  // deferred rows: add each row's segments in order
+    auto row_sum = [&](int ri) {
       float v = 0.f;
       for (int k = 0; k < p.spr; ++k) v += seg[ri * p.spr + k];
-      epi.store(p.r0 + ri, v);
+      return v;
+    };
+    const int nr = p.r1 - p.r0;
+    for (int q = tid; q * p.gran < nr; q += kConsumerThreads) {
+      if (p.gran == 2) epi.store_pair(p.r0 + 2 * q, row_sum(2 * q), row_sum(2 * q + 1));
+      else epi.store(p.r0 + q, row_sum(q));
     }
     named_bar_sync(kBarConsumers, kConsumerThreads);
   }
@@ -538,8 +559,9 @@ __device__ __forceinline__ float warp_sum_transposed(float (&v)[N], int lane) {
 
 // R rows of a stage (row r at w + r * ncols, ncols floats) times kB vectors
 // (vector b at x + b * vs): every weight float4 read from shared memory meets
-// all kB vectors, every x float4 all R rows. put(r, b, value) is called by
-// the lane that holds the sum of row r with vector b.
+// all kB vectors, every x float4 all R rows. put(r, b, value, next) is called
+// by the lane that holds the sum of row r with vector b; next is the sum of
+// row r + 1 with vector b when r + 1 < R.
 template <int R, int kB, class Put>
 __device__ __forceinline__ void rows_times_vectors(const float* w, int ncols, const float* x,
                                                    int vs, int lane, Put put) {
@@ -583,14 +605,17 @@ __device__ __forceinline__ void rows_times_vectors(const float* w, int ncols, co
   for (int i = 0; i < N; ++i)
     v[i] = i >= R * kB ? 0.f : kWide ? (acc[i][0] + acc[i][A > 1 ? 1 : 0]) + (acc[i][A > 2 ? 2 : 0] + acc[i][A > 3 ? 3 : 0]) : acc[i][0];
   const float t = warp_sum_transposed<N>(v, lane);
+  // the next row's sum for the same vector, for paired rows
+  const float tn = __shfl_down_sync(0xffffffffu, t, kB * (32 / N));
   const int idx = lane / (32 / N);
-  if (lane % (32 / N) == 0 && idx < R * kB) put(idx / kB, idx % kB, t);
+  if (lane % (32 / N) == 0 && idx < R * kB) put(idx / kB, idx % kB, t, tn);
 }
 
 // consume_phase for kB input vectors at once (vector b at xs + b * vs): the
 // same stages, each weight read once from the ring for all kB products.
-// epi.store_b(row, b, value) receives row `row` times vector b. Rows longer
-// than a stage leave kB partials per segment in seg, added in segment order.
+// epi.store_b(row, b, value) receives row `row` times vector b, or
+// epi.store_pair_b(row, b, value, value of row + 1) paired rows. Deferred rows
+// leave kB partials per segment in seg, added in segment order.
 template <int kB, class Epi>
 __device__ inline bool consume_phase_b(const Ring& r, uint32_t& g, const StagePlan& p,
                                        const float* xs, int vs, float* seg, Epi& epi, int* err,
@@ -612,10 +637,14 @@ __device__ inline bool consume_phase_b(const Ring& r, uint32_t& g, const StagePl
     const int part = j % p.spr;
     int ri = 0;
     auto put_at = [&](int r0) {
-      return [&, r0](int rr, int b, float v) {
+      return [&, r0](int rr, int b, float v, float vn) {
         const int row = s.row + r0 + rr;
-        if (p.spr > 1) seg[((row - p.r0) * p.spr + part) * kB + b] = v;
-        else epi.store_b(row, b, v);
+        if (p.defer) seg[((row - p.r0) * p.spr + part) * kB + b] = v;
+        else if (p.gran == 2) {
+          if ((rr & 1) == 0) epi.store_pair_b(row, b, v, vn);
+        } else {
+          epi.store_b(row, b, v);
+        }
       };
     };
     for (; ri + 4 <= s.nrows; ri += 4)
@@ -634,12 +663,19 @@ __device__ inline bool consume_phase_b(const Ring& r, uint32_t& g, const StagePl
     if (tid == 0) *s_abort = 1;
     return false;
   }
-  if (p.spr > 1) {  // rows longer than a stage: add the segments in order
-    for (int q = tid; q < (p.r1 - p.r0) * kB; q += kConsumerThreads) {
-      const int ri = q / kB, b = q - ri * kB;
+  if (p.defer) {  // deferred rows: add each row's segments in order
+    auto row_sum = [&](int ri, int b) {
       float v = 0.f;
       for (int k = 0; k < p.spr; ++k) v += seg[(ri * p.spr + k) * kB + b];
-      epi.store_b(p.r0 + ri, b, v);
+      return v;
+    };
+    const int nq = (p.r1 - p.r0) / p.gran;
+    for (int q = tid; q < nq * kB; q += kConsumerThreads) {
+      const int qi = q / kB, b = q - qi * kB;
+      if (p.gran == 2)
+        epi.store_pair_b(p.r0 + 2 * qi, b, row_sum(2 * qi, b), row_sum(2 * qi + 1, b));
+      else
+        epi.store_b(p.r0 + qi, b, row_sum(qi, b));
     }
     named_bar_sync(kBarConsumers, kConsumerThreads);
   }
@@ -649,6 +685,10 @@ __device__ inline bool consume_phase_b(const Ring& r, uint32_t& g, const StagePl
 struct EpiStore {
   float* out;
   __device__ __forceinline__ void store(int row, float v) { out[row] = v; }
+  __device__ __forceinline__ void store_pair(int row, float v0, float v1) {
+    out[row] = v0;
+    out[row + 1] = v1;
+  }
 };
 
 }  // namespace tvl

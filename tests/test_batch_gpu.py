@@ -52,7 +52,9 @@ def batch_greedy_check(m, refs, starts, n_steps, start_pos=0, label=""):
     dict(n_kv_heads=2),                       # grouped query heads
     dict(dim=96, n_heads=2, n_kv_heads=2, hidden_dim=8200, vocab_size=333),  # W2 rows: 2 stages
     dict(n_layers=0),                         # embedding -> final norm -> classifier
-], ids=["base", "gqa2", "wide_ffn", "L0"])
+    dict(dim=2080, n_heads=65, n_kv_heads=65, hidden_dim=64, vocab_size=100, n_layers=1,
+         max_seq=24),                         # W1/W3 row pair wider than a stage
+], ids=["base", "gqa2", "wide_ffn", "L0", "pair_defer"])
 def test_batch_teacher_forced_and_greedy(tvl, B, kw):
     cfg = small_config(max_batch=4, **kw)
     blob = synth.make_blob(cfg, seed=31)

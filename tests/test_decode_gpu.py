@@ -51,7 +51,11 @@ def test_tiny_model_64_steps(tvl):
     dict(n_layers=1, hidden_dim=36, dim=32, n_heads=1, n_kv_heads=1, vocab_size=7),  # one head
     dict(dim=96, n_heads=2, n_kv_heads=2, hidden_dim=8200, vocab_size=333),  # W2 rows: 2 stages
     dict(dim=128, n_heads=1, n_kv_heads=1, hidden_dim=256),  # head_dim 128
-], ids=["base", "gqa2", "mqa", "L0", "v7", "wide_ffn", "hd128"])
+    # rows of 2080 floats: a W1/W3 row pair does not fit one 16 KB stage, so
+    # the pair's two results meet at the end of the phase
+    dict(dim=2080, n_heads=65, n_kv_heads=65, hidden_dim=64, vocab_size=100, n_layers=1,
+         max_seq=24),
+], ids=["base", "gqa2", "mqa", "L0", "v7", "wide_ffn", "hd128", "pair_defer"])
 def test_small_shapes_match_oracle(tvl, kw):
     cfg = small_config(**kw)
     blob = synth.make_blob(cfg, seed=21)
