@@ -71,7 +71,7 @@ SmemPlan plan_smem(int d, int F, int hd, int H, int nch_cap, int max_bytes, int 
   const int att_floats = 3 * hd + kAttMaxChunk + 4 * kConsumerThreads + nch_cap * (hd + 2) + 16;
   // every region is a multiple of 128 bytes, so every region starts aligned
   const int xs = (int)a128(4LL * B * d), vec = (int)a128(4LL * B * std::max(d, F));
-  const int seg = (int)a128(kMaxSegParts * 4), att = (int)a128(4LL * att_floats), misc = 512;
+  const int seg = (int)a128(kMaxSegParts * 4), att = (int)a128(4LL * att_floats), misc = kMiscBytes;
   const int bars = (int)a128(kRingBarBytes);
   const int other = bars + xs + vec + seg + att + misc;
   int nst = (max_bytes - other) / kStageBytes;

@@ -38,6 +38,10 @@ constexpr int kAttMinChunk = 32;    // positions per attention work item, at lea
 constexpr int kAttMaxChunk = 1024;  // and at most
 constexpr int kPhasesPerLayer = 5;  // exchanges per layer: qkv, att, o, h13, f
 constexpr int kMaxBatch = 4;        // sequences one launch can decode together
+// The small shared region of the decode kernel: the abort flag (word 0),
+// reduction scratch (floats 8..39, ints 80..87), the five stage plans.
+constexpr int kPlansOffset = 512;
+constexpr int kMiscBytes = 1024;
 constexpr uint32_t kRefillDelayNs = 1000;  // producer pause before refilling freed stages
 
 struct DecodeArgs {
@@ -697,34 +701,40 @@ __device__ inline bool reduce_candidates(const DecodeArgs& a, int parity, unsign
 
 // ---- the kernel --------------------------------------------------------------------
 
+static_assert(kPlansOffset + 5 * sizeof(StagePlan) <= kMiscBytes, "stage plans overflow");
+
+// This CTA's stage plans of the five GEMV kinds — [Wq|Wk|Wv], Wo, W1/W3
+// (interleaved row pairs), W2, the classifier — the same in every layer and
+// step, so they are worked out once per launch (8-bit rows are 4 + K/4 words).
+template <bool kQ8>
+__device__ inline void phase_plans(const DecodeArgs& a, int c, StagePlan* plans) {
+  const int kd = kQ8 ? 4 + a.d / 4 : a.d, kf = kQ8 ? 4 + a.F / 4 : a.F;
+  plans[0] = plan_stages(a.d + 2 * a.kvd, kd, a.G, c);
+  plans[1] = plan_stages(a.d, kd, a.G, c);
+  plans[2] = plan_stages(2 * a.F, kd, a.G, c, 2);
+  plans[3] = plan_stages(a.d, kf, a.G, c);
+  plans[4] = plan_stages(a.V, kd, a.G, c);
+}
+
 // The weight stream of one launch, in consumption order: per step, each
-// layer's [Wq|Wk|Wv], Wo, W1/W3 (interleaved rows), W2, then the classifier;
-// this CTA's rows.
+// layer's [Wq|Wk|Wv], Wo, W1/W3, W2, then the classifier; this CTA's rows.
 template <bool kQ8>
 struct DecodeSched {
   const DecodeArgs* a;
+  const StagePlan* plans;
   uint32_t refill_delay_ns = kRefillDelayNs;
   int s = 0, l = 0, k = 0;
   __device__ bool next(const float*& W, StagePlan& p) {
     if (s >= a->n_steps) return false;
-    const int c = blockIdx.x;
     if (l < a->L) {
       const unsigned char* lw = a->layer0 + (size_t)l * a->layer_stride;
       const unsigned char* ql = kQ8 ? a->q_layer0 + (size_t)l * a->q_stride : nullptr;
-      // 8-bit rows are 4 + K/4 words in the stages
-      if (k == 0) {
-        W = reinterpret_cast<const float*>(kQ8 ? ql + a->q_wqkv : lw + a->o_wqkv);
-        p = plan_stages(a->d + 2 * a->kvd, kQ8 ? 4 + a->d / 4 : a->d, a->G, c);
-      } else if (k == 1) {
-        W = reinterpret_cast<const float*>(kQ8 ? ql + a->q_wo : lw + a->o_wo);
-        p = plan_stages(a->d, kQ8 ? 4 + a->d / 4 : a->d, a->G, c);
-      } else if (k == 2) {
-        W = reinterpret_cast<const float*>(kQ8 ? ql + a->q_w13 : lw + a->o_w13);
-        p = plan_stages(2 * a->F, kQ8 ? 4 + a->d / 4 : a->d, a->G, c, 2);
-      } else {
-        W = reinterpret_cast<const float*>(kQ8 ? ql + a->q_w2 : lw + a->o_w2);
-        p = plan_stages(a->d, kQ8 ? 4 + a->F / 4 : a->F, a->G, c);
-      }
+      const long long off = k == 0 ? (kQ8 ? a->q_wqkv : a->o_wqkv)
+                            : k == 1 ? (kQ8 ? a->q_wo : a->o_wo)
+                            : k == 2 ? (kQ8 ? a->q_w13 : a->o_w13)
+                                     : (kQ8 ? a->q_w2 : a->o_w2);
+      W = reinterpret_cast<const float*>((kQ8 ? ql : lw) + off);
+      p = plans[k];
       if (++k == 4) {
         k = 0;
         ++l;
@@ -732,7 +742,7 @@ struct DecodeSched {
       return true;
     }
     W = kQ8 ? reinterpret_cast<const float*>(a->q_cls) : a->Wcls;
-    p = plan_stages(a->V, kQ8 ? 4 + a->d / 4 : a->d, a->G, c);
+    p = plans[4];
     l = 0;
     k = 0;
     ++s;
@@ -752,6 +762,7 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
   float* asm_ = reinterpret_cast<float*>(smem + a.sm_att);
   float* red = reinterpret_cast<float*>(smem + a.sm_misc) + 8;
   int* redi = reinterpret_cast<int*>(smem + a.sm_misc) + 80;
+  const StagePlan* plans = reinterpret_cast<const StagePlan*>(smem + a.sm_misc + kPlansOffset);
   const int tid = threadIdx.x, c = blockIdx.x;
   const int vs = kB == 1 ? 0 : a.vs;
   // 16-byte polls in flight per thread: one batch covers a 768-wide vector,
@@ -866,10 +877,10 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
         // partials take el + 1)
         const int M = k == 0 ? a.d + 2 * a.kvd : k == 2 ? 2 * a.F : a.d;
         const int K = k == 3 ? a.F : a.d;
-        const StagePlan plan = plan_stages(M, kQ8 ? 4 + K / 4 : K, a.G, c, k == 2 ? 2 : 1);
+        const StagePlan plan = plans[k];
         unsigned long long* out = k == 0 ? a.x_qkv : k == 1 ? a.x_o : k == 2 ? a.x_h13 : a.x_f;
         EpiTag e{out, el + (k == 0 ? 0u : (unsigned)k + 1u), k == 2 ? a.F : M, k == 2};
-        if constexpr (kB == 1) {
+        if constexpr (kQ8) {
           if (!consume_phase<false, kQ8>(r, g, plan, vec, 1, K, seg, e, a.err, a.err_host,
                                          s_abort))
             return false;
@@ -895,13 +906,12 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
     }
     EpiArgmax<kB> ea{a.logits, a.V};
     ea.init();
-    if constexpr (kB == 1) {
-      if (!consume_phase<false, kQ8>(r, g, plan_stages(a.V, kQ8 ? 4 + a.d / 4 : a.d, a.G, c),
-                                     vec, 1, a.d, seg, ea, a.err, a.err_host, s_abort))
+    if constexpr (kQ8) {
+      if (!consume_phase<false, kQ8>(r, g, plans[4], vec, 1, a.d, seg, ea, a.err, a.err_host,
+                                     s_abort))
         return false;
     } else {
-      if (!consume_phase_b<kB>(r, g, plan_stages(a.V, a.d, a.G, c), vec, vs, seg, ea, a.err,
-                               a.err_host, s_abort))
+      if (!consume_phase_b<kB>(r, g, plans[4], vec, vs, seg, ea, a.err, a.err_host, s_abort))
         return false;
     }
 #pragma unroll
@@ -947,6 +957,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
       r.seq[i] = 0;
     }
     *s_abort = 0;
+    phase_plans<kQ8>(a, blockIdx.x, reinterpret_cast<StagePlan*>(smem + a.sm_misc + kPlansOffset));
     fence_mbar_init();
   }
   __syncthreads();
@@ -954,6 +965,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
     if (threadIdx.x == kConsumerThreads) {
       DecodeSched<kQ8> sched;
       sched.a = &a;
+      sched.plans = reinterpret_cast<const StagePlan*>(smem + a.sm_misc + kPlansOffset);
       run_producer(r, sched, a.err, a.err_host, s_abort);
     }
     return;

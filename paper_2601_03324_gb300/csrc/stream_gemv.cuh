@@ -649,12 +649,13 @@ __device__ inline bool consume_phase_b(const Ring& r, uint32_t& g, const StagePl
     };
     for (; ri + 4 <= s.nrows; ri += 4)
       rows_times_vectors<4, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, put_at(ri));
-    if (ri + 2 <= s.nrows) {
+    if (s.nrows - ri == 3) {
+      rows_times_vectors<3, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, put_at(ri));
+    } else if (s.nrows - ri == 2) {
       rows_times_vectors<2, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, put_at(ri));
-      ri += 2;
-    }
-    if (ri < s.nrows)
+    } else if (s.nrows - ri == 1) {
       rows_times_vectors<1, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, put_at(ri));
+    }
     __syncwarp();
     if (lane == 0) mbar_arrive(&r.empty[slot]);  // stage free for the producer
   }
