@@ -522,17 +522,23 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
     const int gi = tid / hd4, f = tid - gi * hd4;
     const int n = t1 - t0;
     const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
-    float4 kr0 = z4, kr1 = z4, v0 = z4, v1 = z4;
+    // the first three K and V rows of each thread, loaded before q is ready
+    float4 kr0 = z4, kr1 = z4, kr2 = z4, v0 = z4, v1 = z4, v2 = z4;
     {
       const int tk = t0 + warp * ppw + sub;
       if (li < hd4 && tk < t1 && tk != pos)
         kr0 = ldcg4(reinterpret_cast<const float4*>(kbase + (size_t)tk * a.kvd) + li);
       if (li < hd4 && tk + pstride < t1 && tk + pstride != pos)
         kr1 = ldcg4(reinterpret_cast<const float4*>(kbase + (size_t)(tk + pstride) * a.kvd) + li);
+      if (li < hd4 && tk + 2 * pstride < t1 && tk + 2 * pstride != pos)
+        kr2 = ldcg4(reinterpret_cast<const float4*>(kbase + (size_t)(tk + 2 * pstride) * a.kvd) +
+                    li);
       if (gi < ng && gi < n && t0 + gi != pos)
         v0 = ldcg4(reinterpret_cast<const float4*>(vbase + (size_t)(t0 + gi) * a.kvd) + f);
       if (gi < ng && gi + ng < n && t0 + gi + ng != pos)
         v1 = ldcg4(reinterpret_cast<const float4*>(vbase + (size_t)(t0 + gi + ng) * a.kvd) + f);
+      if (gi < ng && gi + 2 * ng < n && t0 + gi + 2 * ng != pos)
+        v2 = ldcg4(reinterpret_cast<const float4*>(vbase + (size_t)(t0 + gi + 2 * ng) * a.kvd) + f);
     }
     // q (and the new k, v) with RoPE: pair i turns by pos * theta^(-2i/hd).
     // Pair i of a head is one 16-byte tagged load.
@@ -556,20 +562,21 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
       }
     }
     if (!vote_ok(ok, pc.s_abort)) return false;
-    if (has_new && (h % group) == 0) {  // one writer per kv head
+    const bool kv_writer = has_new && (h % group) == 0;  // one writer per kv head
+    if (kv_writer) {  // thread j < hd writes element j of the new K and V rows
       float* kd = a.kc + lay + (size_t)pos * a.kvd + kvh * hd;
       float* vd = a.vc + lay + (size_t)pos * a.kvd + kvh * hd;
-      for (int j = tid; j < hd; j += kConsumerThreads) {
-        kd[j] = kp[j];
-        vd[j] = vp[j];
+      if (tid < hd) {
+        kd[tid] = kp[tid];
+        vd[tid] = vp[tid];
       }
-      if (tid < hd) __threadfence();  // cache row visible before this item's partials are
     }
     if (gi < ng && t0 + gi == pos) v0 = reinterpret_cast<const float4*>(vp)[f];
     if (gi < ng && t0 + gi + ng == pos) v1 = reinterpret_cast<const float4*>(vp)[f];
+    if (gi < ng && t0 + gi + 2 * ng == pos) v2 = reinterpret_cast<const float4*>(vp)[f];
     // scores s_t = (q . k_t) * scale for t in [t0, t1); the first pass uses the rows loaded above
     const float4* q4 = reinterpret_cast<const float4*>(q);
-    for (int tb = t0 + warp * ppw, first = 1; tb < t1; tb += 2 * pstride, first = 0) {
+    for (int tb = t0 + warp * ppw, it = 0; tb < t1; tb += 2 * pstride, ++it) {
       float acc[2] = {0.f, 0.f};
 #pragma unroll
       for (int u = 0; u < 2; ++u) {
@@ -579,7 +586,10 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
                                  ? reinterpret_cast<const float4*>(kp)
                                  : reinterpret_cast<const float4*>(kbase + (size_t)t * a.kvd);
           for (int f = li; f < hd4; f += lpp) {
-            const float4 kv = (t == pos) ? k4[f] : first ? (u ? kr1 : kr0) : ldcg4(k4 + f);
+            const float4 kv = (t == pos)             ? k4[f]
+                              : it == 0              ? (u ? kr1 : kr0)
+                              : (it == 1 && u == 0) ? kr2
+                                                     : ldcg4(k4 + f);
             const float4 qv = q4[f];
             acc[u] = fmaf(qv.x, kv.x, acc[u]);
             acc[u] = fmaf(qv.y, kv.y, acc[u]);
@@ -623,13 +633,18 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
       };
       if (gi < n) fma4(sc[gi], v0);
       if (gi + ng < n) fma4(sc[gi + ng], v1);
-      for (int i = gi + 2 * ng; i < n; i += ng) fma4(sc[i], vrow(t0 + i));
+      if (gi + 2 * ng < n) fma4(sc[gi + 2 * ng], v2);
+      for (int i = gi + 3 * ng; i < n; i += ng) fma4(sc[i], vrow(t0 + i));
       reinterpret_cast<float4*>(part)[gi * hd4 + f] = acc;
     }
     named_bar_sync(kBarConsumers, kConsumerThreads);
     float own = 0.f;  // this chunk's sum of e_t v_t, element tid (tid < hd)
     if (tid < hd)
       for (int g2 = 0; g2 < ng; ++g2) own += part[g2 * hd + tid];
+    // Release: the new cache row, written by these threads long before, is
+    // visible before any result of this item (readers in later steps see
+    // the row through the chain of exchanges that starts here).
+    if (kv_writer && tid < hd) __threadfence();
     if (c != 0) {
       unsigned long long* rec = a.x_att + ((size_t)hb * a.nch_cap + c) * a.att_stride;
       if (tid < hd) st_tag(rec + 4 + tid, tag_att, own);
