@@ -576,34 +576,47 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
     if (gi < ng && t0 + gi + 2 * ng == pos) v2 = reinterpret_cast<const float4*>(vp)[f];
     // scores s_t = (q . k_t) * scale for t in [t0, t1); the first pass uses the rows loaded above
     const float4* q4 = reinterpret_cast<const float4*>(q);
-    for (int tb = t0 + warp * ppw, it = 0; tb < t1; tb += 2 * pstride, ++it) {
-      float acc[2] = {0.f, 0.f};
+    {
+      // positions in groups of three rows per lane: row rr of group j is
+      // position t0 + j * 3 * pstride + warp * ppw + sub + rr * pstride; the
+      // first group is the rows loaded above, each later one three loads at once
+      const float4 qv = li < hd4 ? q4[li] : z4;
+      const float4 kn = li < hd4 ? reinterpret_cast<const float4*>(kp)[li] : z4;
+      for (int tg = t0 + warp * ppw + sub; tg - sub < t1; tg += 3 * pstride) {
+        float4 kv[3];
+        if (tg - sub == t0 + warp * ppw) {
+          kv[0] = kr0;
+          kv[1] = kr1;
+          kv[2] = kr2;
+        } else {
 #pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int t = tb + u * pstride + sub;
-        if (t < t1) {
-          const float4* k4 = (t == pos)
-                                 ? reinterpret_cast<const float4*>(kp)
-                                 : reinterpret_cast<const float4*>(kbase + (size_t)t * a.kvd);
-          for (int f = li; f < hd4; f += lpp) {
-            const float4 kv = (t == pos)             ? k4[f]
-                              : it == 0              ? (u ? kr1 : kr0)
-                              : (it == 1 && u == 0) ? kr2
-                                                     : ldcg4(k4 + f);
-            const float4 qv = q4[f];
-            acc[u] = fmaf(qv.x, kv.x, acc[u]);
-            acc[u] = fmaf(qv.y, kv.y, acc[u]);
-            acc[u] = fmaf(qv.z, kv.z, acc[u]);
-            acc[u] = fmaf(qv.w, kv.w, acc[u]);
+          for (int rr = 0; rr < 3; ++rr) {
+            const int t = tg + rr * pstride;
+            kv[rr] = (li < hd4 && t < t1 && t != pos)
+                         ? ldcg4(reinterpret_cast<const float4*>(kbase + (size_t)t * a.kvd) + li)
+                         : z4;
           }
         }
-      }
+        float s3[3];
 #pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int t = tb + u * pstride + sub;
-        float s = acc[u];
-        for (int o = lpp >> 1; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-        if (t < t1 && li == 0) sc[t - t0] = s * a.att_scale;
+        for (int rr = 0; rr < 3; ++rr) {
+          const float4 k = tg + rr * pstride == pos ? kn : kv[rr];
+          float acc = 0.f;
+          acc = fmaf(qv.x, k.x, acc);
+          acc = fmaf(qv.y, k.y, acc);
+          acc = fmaf(qv.z, k.z, acc);
+          acc = fmaf(qv.w, k.w, acc);
+          s3[rr] = acc;
+        }
+        for (int o = lpp >> 1; o > 0; o >>= 1) {
+#pragma unroll
+          for (int rr = 0; rr < 3; ++rr) s3[rr] += __shfl_xor_sync(0xffffffffu, s3[rr], o);
+        }
+#pragma unroll
+        for (int rr = 0; rr < 3; ++rr) {
+          const int t = tg + rr * pstride;
+          if (t < t1 && li == 0) sc[t - t0] = s3[rr] * a.att_scale;
+        }
       }
     }
     auto vrow = [&](int t) -> float4 {
@@ -612,16 +625,32 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
                                                                 kvh * hd) + f);
     };
     named_bar_sync(kBarConsumers, kConsumerThreads);
-    float m = -INFINITY;
-    for (int i = tid; i < n; i += kConsumerThreads) m = fmaxf(m, sc[i]);
-    m = block_max(m, red);
-    float ls = 0.f;
-    for (int i = tid; i < n; i += kConsumerThreads) {
-      const float e = expf(sc[i] - m);
-      sc[i] = e;
-      ls += e;
+    // softmax weights e_t = exp(s_t - m), m = max s_t, and l = sum e_t. A chunk
+    // of at most 64 positions is reduced by every warp on its own (the same
+    // values in every warp, no barrier); a longer one by the whole block,
+    // which leaves e_t in sc.
+    const bool warp_softmax = n <= 64;
+    float m, ls;
+    if (warp_softmax) {
+      const float s0 = lane < n ? sc[lane] : -INFINITY;
+      const float s1 = lane + 32 < n ? sc[lane + 32] : -INFINITY;
+      m = warp_max(fmaxf(s0, s1));
+      const float e0 = lane < n ? expf(s0 - m) : 0.f;
+      const float e1 = lane + 32 < n ? expf(s1 - m) : 0.f;
+      ls = warp_sum(e0 + e1);
+    } else {
+      m = -INFINITY;
+      for (int i = tid; i < n; i += kConsumerThreads) m = fmaxf(m, sc[i]);
+      m = block_max(m, red);
+      ls = 0.f;
+      for (int i = tid; i < n; i += kConsumerThreads) {
+        const float e = expf(sc[i] - m);
+        sc[i] = e;
+        ls += e;
+      }
+      ls = block_sum(ls, red);  // its barriers also publish sc
     }
-    ls = block_sum(ls, red);  // its barriers also publish sc
+    auto weight = [&](int i) { return warp_softmax ? expf(sc[i] - m) : sc[i]; };
     // o = sum_t e_t v_t: thread (gi, f) sums float4 column f over t = gi, gi+ng, ...
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     if (gi < ng) {
@@ -631,10 +660,10 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
         acc.z = fmaf(e, vv.z, acc.z);
         acc.w = fmaf(e, vv.w, acc.w);
       };
-      if (gi < n) fma4(sc[gi], v0);
-      if (gi + ng < n) fma4(sc[gi + ng], v1);
-      if (gi + 2 * ng < n) fma4(sc[gi + 2 * ng], v2);
-      for (int i = gi + 3 * ng; i < n; i += ng) fma4(sc[i], vrow(t0 + i));
+      if (gi < n) fma4(weight(gi), v0);
+      if (gi + ng < n) fma4(weight(gi + ng), v1);
+      if (gi + 2 * ng < n) fma4(weight(gi + 2 * ng), v2);
+      for (int i = gi + 3 * ng; i < n; i += ng) fma4(weight(i), vrow(t0 + i));
       reinterpret_cast<float4*>(part)[gi * hd4 + f] = acc;
     }
     named_bar_sync(kBarConsumers, kConsumerThreads);

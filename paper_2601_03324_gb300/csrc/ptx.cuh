@@ -119,7 +119,16 @@ __device__ __forceinline__ int ld_volatile_s32(const int* p) {
 
 // Loads of data written by other CTAs during this kernel: cached in L2 only.
 __device__ __forceinline__ float ldcg(const float* p) { return __ldcg(p); }
-__device__ __forceinline__ float4 ldcg4(const float4* p) { return __ldcg(p); }
+// An L2 load the compiler keeps where it is written: never executed ahead of
+// the branch that guards it (a plain cache-hinted load may be, and a select
+// then waits for its round trip even when it picks the other operand).
+__device__ __forceinline__ float4 ldcg4(const float4* p) {
+  float4 v;
+  asm volatile("ld.global.cg.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "l"(p));
+  return v;
+}
 
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
