@@ -36,6 +36,8 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "batch-1 decode tokens/s (110M FP32); GEMV HBM GB/s vs ~8 TB/s peak"
+METRIC_BATCH = "decode tokens/s, {b} sequences per step (110M FP32)"
+BATCH_STARTS = [1, 100, 2000, 31999]  # first tokens of the sequences of a batched run
 PAPER_TOKS = 61.3  # the paper's 110M FP32 decode on one M2 Pro core (Table 1)
 SEQ = 256
 FALLBACK_HBM_GBS = 6800.0
@@ -54,6 +56,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--gemv-sweep", action="store_true", help="GEMV GB/s per shape instead")
+    ap.add_argument("--batch", type=int, default=1, choices=[1, 2, 3, 4],
+                    help="sequences decoded together per launch (tvl_decode_greedy_batch)")
     return ap.parse_args()
 
 
@@ -119,12 +123,13 @@ def job_tokens_per_s(world: int, steps: int, max_ms: float) -> float:
     return world * steps / (max_ms * 1e-3)
 
 
-def step_bytes(cfg: dict, streamed: int, pos: int) -> int:
-    """Algorithmic bytes of one step at position pos: every weight once, the
-    K/V cache rows of positions < pos, the new K/V row, the logits."""
+def step_bytes(cfg: dict, streamed: int, pos: int, batch: int = 1) -> int:
+    """Algorithmic bytes of one step at position pos: every weight once (for
+    all sequences of the batch), and per sequence the K/V cache rows of
+    positions < pos, the new K/V row, the logits."""
     d, L, V = cfg["dim"], cfg["n_layers"], cfg["vocab_size"]
     kvd = cfg["n_kv_heads"] * (d // cfg["n_heads"])
-    return streamed + 2 * pos * kvd * 4 * L + 2 * kvd * 4 * L + 4 * V
+    return streamed + batch * (2 * pos * kvd * 4 * L + 2 * kvd * 4 * L + 4 * V)
 
 
 class Clocks:
@@ -245,7 +250,7 @@ def run_reference(args, cfg, rank, world):
     return 0
 
 
-def workload_config(name, cfg):
+def workload_config(name, cfg, batch=1):
     desc = {"110m": "110M Llama-2-shape FP32 decoder (d768 L12 H12 F2048 V32000, tied), "
                     "batch 1, greedy 256-step sequences from token 1",
             "110m-long": "110M Llama-2-shape FP32 decoder (d768 L12 H12 F2048 V32000, tied), "
@@ -256,7 +261,10 @@ def workload_config(name, cfg):
             "7b": "7B Llama-2-shape FP32 decoder (d4096 L32 H32 F11008 V32000, untied), batch 1, "
                   "greedy 16-step sequences from token 1"}[name]
     seq = 128 if name == "110m-long" else min(cfg["steps"], cfg["max_seq"])
-    return {"workload": desc, "seq_steps": seq, "batch": 1,
+    if batch > 1:
+        desc = desc.replace("batch 1, greedy", f"{batch} sequences per launch (first tokens "
+                            f"{BATCH_STARTS[:batch]}), greedy").replace(" from token 1", "")
+    return {"workload": desc, "seq_steps": seq, "batch": batch,
             "weights_seed": cfg["seed"], "parallelism": "replicas",
             "l2": "inputs larger than L2: every step streams all weights (> L2 size)"}
 
@@ -329,9 +337,16 @@ def main():
     torch.cuda.set_device(local_rank)
     from paper_2601_03324_gb300 import tvl
 
+    B = args.batch
+    if B > 1 and (args.weights != "f32" or args.workload == "110m-long"):
+        print(json.dumps({"error": "--batch > 1 needs --weights f32 and a workload other than "
+                                   "110m-long"}))
+        return 2
     blob = synth.make_blob(cfg)
     if args.weights == "q8":
         cfg = dict(cfg, weight_bits=8)
+    if B > 1:
+        cfg = dict(cfg, max_batch=B)
     stream = torch.cuda.Stream()
     model = tvl.Model(cfg, blob, stream=stream.cuda_stream)
     info = model.info()
@@ -356,7 +371,10 @@ def main():
             if events is not None:
                 e0 = torch.cuda.Event(enable_timing=True)
                 e0.record(stream)
-            model.decode_greedy(tok0, pos0, n, tokens=False)
+            if B == 1:
+                model.decode_greedy(tok0, pos0, n, tokens=False)
+            else:
+                model.decode_greedy_batch(BATCH_STARTS[:B], pos0, n, tokens=False)
             if events is not None:
                 e1 = torch.cuda.Event(enable_timing=True)
                 e1.record(stream)
@@ -395,36 +413,45 @@ def main():
     full = [(a.elapsed_time(b), n) for (a, b, n) in ev]
     launch_ms = statistics.mean(t for t, n in full)
     n_typ = full[0][1]
-    bytes_launch = sum(step_bytes(cfg, info.streamed_bytes, pos0 + p) for p in range(n_typ))
+    bytes_launch = sum(step_bytes(cfg, info.streamed_bytes, pos0 + p, B) for p in range(n_typ))
     peak, peak_src = measured_peaks()
     achieved = bytes_launch / (statistics.mean(t for t, n in full if n == n_typ) * 1e-3) / 1e9
-    traffic = committed_traffic(args.workload + ("_q8" if args.weights == "q8" else ""),
-                                bytes_launch)
+    traffic = committed_traffic(args.workload + ("_q8" if args.weights == "q8" else "") +
+                                (f"_b{B}" if B > 1 else ""), bytes_launch)
     steps_ns = model.step_times(n_typ).astype(np.float64)
     dts = np.diff(steps_ns) / 1e3 if n_typ > 1 else np.array([launch_ms * 1e3])
 
-    # end to end through the public API: token in, host logits out, host argmax
+    # end to end through the public API: token(s) in, host logits out, host argmax
     e2e = None
     if not args.no_e2e:
         import torch as _t
-        host_logits = _t.empty(cfg["vocab_size"], dtype=_t.float32, pin_memory=True).numpy()
+        host_logits = _t.empty(B * cfg["vocab_size"], dtype=_t.float32, pin_memory=True).numpy()
+        V = cfg["vocab_size"]
         k_e2e = min(args.steps, 2048)
-        tok = tok0
+        first = [tok0] if B == 1 else BATCH_STARTS[:B]
+
+        def api_step(toks, p):
+            if B == 1:
+                model.forward(toks[0], p, host_logits)
+            else:
+                model.forward_batch(toks, p, host_logits)
+            return [int(np.argmax(host_logits[b * V:(b + 1) * V])) for b in range(B)]
+
+        toks = list(first)
         for p in range(pos0, pos0 + 8):
-            model.forward(tok, p, host_logits)
-            tok = int(np.argmax(host_logits))
+            toks = api_step(toks, p)
         t0 = time.perf_counter()
-        tok, pos = tok0, pos0
-        for s in range(k_e2e):
-            model.forward(tok, pos, host_logits)
-            tok = int(np.argmax(host_logits))
+        toks, pos = list(first), pos0
+        for s_ in range(k_e2e):
+            toks = api_step(toks, pos)
             pos += 1
             if pos == pos0 + seq:
-                tok, pos = tok0, pos0
+                toks, pos = list(first), pos0
         e2e_s = time.perf_counter() - t0
-        e2e = {"value": world * k_e2e / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": 4,
-               "d2h_bytes_per_step": 4 * cfg["vocab_size"],
-               "note": "tvl_forward per step: token as launch argument, logits to pinned host "
+        e2e = {"value": world * B * k_e2e / e2e_s, "unit": "tokens/s",
+               "h2d_bytes_per_step": 4 * B, "d2h_bytes_per_step": 4 * B * V,
+               "note": ("tvl_forward" if B == 1 else "tvl_forward_batch") +
+                       " per step: token(s) as launch arguments, logits to pinned host "
                        "memory, argmax on the host"}
 
     cpu = None
@@ -435,15 +462,17 @@ def main():
                "sample": f"first {n} greedy steps of the workload from token 1 "
                          f"({el:.1f} s, double accumulators, one thread)"}
 
-    value = job_tokens_per_s(world, args.steps, el_ms)
+    value = job_tokens_per_s(world, args.steps, el_ms) * B
     line = {
-        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "metric": METRIC if B == 1 else METRIC_BATCH.format(b=B), "value": value,
+        "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": el_ms / args.steps,
         "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": value / PAPER_TOKS if args.workload == "110m" and args.weights == "f32" else None,
+        "vs_baseline": (value / PAPER_TOKS
+                        if args.workload == "110m" and args.weights == "f32" and B == 1 else None),
         "dtype": "f32" if args.weights == "f32" else "f32 activations, int8 weight rows",
         "data": "synthetic (seeded N(0, 0.02) weights)",
-        "config": dict(workload_config(args.workload, cfg), weights=args.weights),
+        "config": dict(workload_config(args.workload, cfg, B), weights=args.weights),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "kernel": "decode_kernel", "peak_source": peak_src,
