@@ -168,15 +168,21 @@ class Clocks:
             try:
                 ts = time.mktime(time.strptime(parts[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
                 ts += float("0." + parts[0].split(".")[1]) if "." in parts[0] else 0.0
-                rows.append((ts, float(parts[1]), float(parts[2]), parts[5:9]))
+                try:
+                    pw = float(parts[3])
+                except ValueError:
+                    pw = None
+                rows.append((ts, float(parts[1]), float(parts[2]), parts[5:9], pw))
             except (ValueError, IndexError):
                 continue
         win = [r for r in rows if t0 - 0.06 <= r[0] <= t1 + 0.06] or rows[-3:]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         reasons = sorted({names[i] for r in win for i, v in enumerate(r[3]) if v == "Active"})
+        pws = [r[4] for r in win if r[4] is not None]
         return {"sm_mhz": statistics.median([r[1] for r in win]) if win else None,
                 "sm_max_mhz": max(r[2] for r in win) if win else None,
-                "reasons": reasons, "samples": len(win)}
+                "reasons": reasons, "samples": len(win),
+                "power_w": statistics.median(pws) if pws else None}
 
 
 def cpu_oracle_rate(cfg, blob, seconds: float, weight_bits: int = 0):
@@ -463,6 +469,13 @@ def main():
                          f"({el:.1f} s, double accumulators, one thread)"}
 
     value = job_tokens_per_s(world, args.steps, el_ms) * B
+    # board energy per token (paper's energy section reports mJ/token): the
+    # median board power sampled during the timed region times its duration
+    energy = None
+    if clk.get("power_w"):
+        energy = {"power_w": clk["power_w"],
+                  "mj_per_token": 1e3 * clk["power_w"] * (el_ms * 1e-3) / (args.steps * B),
+                  "note": "nvidia-smi power.draw (board), median over the timed region"}
     line = {
         "metric": METRIC if B == 1 else METRIC_BATCH.format(b=B), "value": value,
         "unit": "tokens/s", "n_gpus": world,
@@ -483,7 +496,12 @@ def main():
         "gpu_launches": launches,
         "clocks": clk,
         "step_latency_us": {"p50": float(np.percentile(dts, 50)),
-                            "p99": float(np.percentile(dts, 99))},
+                            "p90": float(np.percentile(dts, 90)),
+                            "p99": float(np.percentile(dts, 99)),
+                            "max": float(np.max(dts)), "std": float(np.std(dts)),
+                            "source": "device timestamps at the end of each step of one "
+                                      "launch (tvl_step_times)"},
+        "energy": energy,
         "grid": info.grid, "ring_stages": info.ring_stages,
     }
     if rank == 0:
