@@ -138,6 +138,22 @@ tvl_status tvl_forward_batch(tvl_model* m, int32_t batch, const int32_t* tokens,
 tvl_status tvl_decode_greedy_batch(tvl_model* m, int32_t batch, const int32_t* start_tokens,
                                    int32_t start_pos, int32_t n_steps, int32_t* tokens_out);
 
+/* Multi-token prefill of sequence slot 0: tokens[0..n) (host array) at
+ * positions start_pos .. start_pos + n - 1 run through every layer as one
+ * block of n rows per layer, writing their K/V rows into the cache, and the
+ * logits of the last position are returned — the same computation as n
+ * tvl_forward calls (§2.1, §7.1), with each layer's weights read once for all
+ * n positions. The products with the weight matrices run as float32 GEMMs in
+ * cuBLAS; the first call allocates the activations for max_seq positions
+ * (and a cuBLAS handle), kept until tvl_free. Positions 0 .. start_pos - 1
+ * must hold this sequence's K/V already.
+ *   logits_out: V floats, as for tvl_forward (device: no wait; host: waits;
+ *   NULL: kept on the device).
+ *   n >= 1, start_pos >= 0, start_pos + n <= max_seq, tokens in [0, V), else
+ *   TVL_E_RANGE; a model loaded with weight_bits 8: TVL_E_UNSUPPORTED. */
+tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n, int32_t start_pos,
+                       float* logits_out);
+
 /* Standalone GEMV y = W x (§6.1), W [d_out x d_in] row-major, x [d_in],
  * y [d_out]; all device pointers; queued on `stream` (NULL = default stream),
  * does not wait. d_out >= 1, d_in >= 1, else TVL_E_INVAL. The fast path

@@ -13,33 +13,10 @@
 
 #include "decode_kernel.cuh"
 #include "host_common.h"
+#include "model.h"
 
 using namespace tvl;
 
-struct tvl_model {
-  tvl_config cfg{};
-  bool tied = false;
-  int device = 0;
-  cudaStream_t stream = nullptr;
-  bool own_stream = false;
-  unsigned char* arena = nullptr;
-  size_t arena_bytes = 0;
-  size_t weight_bytes = 0;
-  int64_t streamed_bytes = 0;
-  DecodeArgs args{};
-  int max_batch = 1;
-  // per batch size B = 1..max_batch: the kernel (decode_kernel<q8, B>), its
-  // shared-memory plan and the words between two sequences' phase inputs
-  const void* kernel[kMaxBatch + 1] = {};
-  struct Plan {
-    int sm_ring, sm_bars, sm_xs, sm_vec, sm_seg, sm_att, sm_misc, nst, total;
-  } plan[kMaxBatch + 1] = {};
-  int vs = 0;
-  int smem_bytes = 0;
-  int* err_host = nullptr;  // pinned, mapped: the kernel writes its error code here too
-  unsigned epoch = 1;       // tag of the next launch's first exchange (0 = never written)
-  tvl_status sticky = TVL_OK;
-};
 
 namespace tvl {
 
@@ -119,6 +96,7 @@ tvl_status check_device_error(tvl_model* m) {
 
 void destroy(tvl_model* m) {
   if (!m) return;
+  prefill_release(m);
   if (m->arena) cudaFree(m->arena);
   if (m->err_host) cudaFreeHost(m->err_host);
   if (m->own_stream && m->stream) cudaStreamDestroy(m->stream);

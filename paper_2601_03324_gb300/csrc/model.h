@@ -1,0 +1,40 @@
+// model.h — the loaded-model state shared by the library's host files
+// (decode.cu: loading and decode launches; prefill.cu: multi-token prefill).
+#pragma once
+#include "decode_kernel.cuh"
+#include "host_common.h"
+
+using tvl::DecodeArgs;
+using tvl::kMaxBatch;
+
+struct tvl_model {
+  tvl_config cfg{};
+  bool tied = false;
+  int device = 0;
+  cudaStream_t stream = nullptr;
+  bool own_stream = false;
+  unsigned char* arena = nullptr;
+  size_t arena_bytes = 0;
+  size_t weight_bytes = 0;
+  int64_t streamed_bytes = 0;
+  DecodeArgs args{};
+  int max_batch = 1;
+  // per batch size B = 1..max_batch: the kernel (decode_kernel<q8, B>), its
+  // shared-memory plan and the words between two sequences' phase inputs
+  const void* kernel[kMaxBatch + 1] = {};
+  struct Plan {
+    int sm_ring, sm_bars, sm_xs, sm_vec, sm_seg, sm_att, sm_misc, nst, total;
+  } plan[kMaxBatch + 1] = {};
+  int vs = 0;
+  int smem_bytes = 0;
+  int* err_host = nullptr;  // pinned, mapped: the kernel writes its error code here too
+  unsigned epoch = 1;       // tag of the next launch's first exchange (0 = never written)
+  tvl_status sticky = TVL_OK;
+  // multi-token prefill (prefill.cu): created on first use
+  void* blas = nullptr;  // cublasHandle_t bound to `stream`
+  float* pf = nullptr;   // activations of up to max_seq positions
+  size_t pf_bytes = 0;
+};
+
+// Releases what prefill created (prefill.cu).
+void prefill_release(tvl_model* m);

@@ -64,6 +64,8 @@ def _load():
     L.tvl_forward.argtypes = [P, i32, i32, P]
     L.tvl_decode_greedy.restype = st
     L.tvl_decode_greedy.argtypes = [P, i32, i32, i32, P]
+    L.tvl_prefill.restype = st
+    L.tvl_prefill.argtypes = [P, P, i32, i32, P]
     L.tvl_forward_batch.restype = st
     L.tvl_forward_batch.argtypes = [P, i32, P, i32, P]
     L.tvl_decode_greedy_batch.restype = st
@@ -98,7 +100,7 @@ def _load():
 lib = _load()
 
 EXPORTED = ["tvl_blob_bytes", "tvl_load", "tvl_load_file", "tvl_forward", "tvl_decode_greedy",
-            "tvl_forward_batch", "tvl_decode_greedy_batch",
+            "tvl_forward_batch", "tvl_decode_greedy_batch", "tvl_prefill",
             "tvl_gemv", "tvl_gemv_noalloc", "tvl_q8_bytes", "tvl_quantize_q8", "tvl_gemv_q8",
             "tvl_sync", "tvl_free", "tvl_status_string", "tvl_last_error",
             "tvl_get_info", "tvl_step_times", "tvl_selftest_barrier_timeout"]
@@ -221,6 +223,20 @@ class Model:
         _check(lib.tvl_decode_greedy(self._h, int(start_token), int(start_pos), int(n_steps),
                                      ptr), "tvl_decode_greedy")
         return out
+
+    def prefill(self, tokens, start_pos: int = 0, logits=None):
+        """Prefill: len(tokens) positions from start_pos in one pass per layer;
+        logits of the last position as for forward()."""
+        toks = np.ascontiguousarray(tokens, dtype=np.int32)
+        if logits is None:
+            ptr = None
+        else:
+            if isinstance(logits, np.ndarray):
+                assert logits.dtype == np.float32 and logits.size >= self.vocab
+            ptr = ctypes.c_void_p(_addr(logits))
+        _check(lib.tvl_prefill(self._h, ctypes.c_void_p(toks.ctypes.data), int(toks.size),
+                               int(start_pos), ptr), "tvl_prefill")
+        return logits
 
     def forward_batch(self, tokens, pos: int, logits=None):
         """One step of len(tokens) sequences at position pos. logits: None,
