@@ -228,6 +228,56 @@ __device__ inline bool poll_pairs_at(int npairs, Addr addr, unsigned tag, const 
   return true;
 }
 
+// Poll quads j = tid, tid + 224, ... (nquads quads of four consecutive words),
+// Q quads (2 Q 16-byte loads) in flight per thread, and load quad j mod n4 of
+// aux (the RMSNorm gains) for each while the polls are out; fn(j, v, aux quad)
+// takes each ready quad. Returns false if this thread gave up.
+template <int Q, class Fn>
+__device__ inline bool poll_quads(const unsigned long long* src, int nquads, unsigned tag,
+                                  const float4* aux, int n4, const Poll& c, Fn fn) {
+  for (int base = threadIdx.x; base < nquads; base += kConsumerThreads * Q) {
+    ulonglong2 lo[Q], hi[Q];
+    float4 ax[Q];
+    unsigned pending = 0;
+#pragma unroll
+    for (int b = 0; b < Q; ++b) {
+      const int j = base + b * kConsumerThreads;
+      if (j < nquads) {
+        lo[b] = ld_tag2(src + 4 * j);
+        hi[b] = ld_tag2(src + 4 * j + 2);
+        pending |= 1u << b;
+      }
+    }
+#pragma unroll
+    for (int b = 0; b < Q; ++b) {
+      const int j = base + b * kConsumerThreads;
+      if (j < nquads) ax[b] = __ldg(aux + j % n4);
+    }
+    PollClock clk;
+    while (true) {
+#pragma unroll
+      for (int b = 0; b < Q; ++b) {
+        if (((pending >> b) & 1u) && tags_are(lo[b], tag) && tags_are(hi[b], tag)) {
+          fn(base + b * kConsumerThreads,
+             make_float4(lo_f(lo[b].x), lo_f(lo[b].y), lo_f(hi[b].x), lo_f(hi[b].y)), ax[b]);
+          pending &= ~(1u << b);
+        }
+      }
+      if (!pending) break;
+      if (!clk.keep_waiting(c)) return false;
+#pragma unroll
+      for (int b = 0; b < Q; ++b) {
+        if ((pending >> b) & 1u) {
+          const int j = base + b * kConsumerThreads;
+          lo[b] = ld_tag2(src + 4 * j);
+          hi[b] = ld_tag2(src + 4 * j + 2);
+        }
+      }
+    }
+  }
+  return true;
+}
+
 // One pair, re-read until current (used where a thread needs a single pair).
 __device__ inline bool poll_one(const unsigned long long* p, unsigned tag, const Poll& c,
                                 ulonglong2& v) {
@@ -298,103 +348,16 @@ __device__ inline void block_argmax(float& v, int& idx, float* redv, int* redi) 
   named_bar_sync(kBarConsumers, kConsumerThreads);
 }
 
-// Sums over the consumer threads of kB values at once (one barrier pair);
-// red holds 7 * kB floats. Every thread gets the totals.
-template <int kB>
-__device__ inline void block_sum_n(float (&v)[kB], float* red) {
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+// The input of a phase that follows an RMSNorm is x * g without the factor
+// r = 1/sqrt(mean x^2 + eps); each row's dot product is multiplied by r here
+// (W ((x * g) r) = r W (x * g)). scale[b] is sequence b's factor, 1 for the
+// phases without a norm.
+__device__ __forceinline__ float pick_scale(const float (&sc)[kMaxBatch], int b) {
+  float v = sc[0];
 #pragma unroll
-  for (int b = 0; b < kB; ++b) {
-    const float t = warp_sum(v[b]);
-    if (lane == 0) red[warp * kB + b] = t;
-  }
-  named_bar_sync(kBarConsumers, kConsumerThreads);
-#pragma unroll
-  for (int b = 0; b < kB; ++b) {
-    float t = 0.f;
-#pragma unroll
-    for (int w = 0; w < kConsumerWarps; ++w) t += red[w * kB + b];
-    v[b] = t;
-  }
-  named_bar_sync(kBarConsumers, kConsumerThreads);
-}
-
-// RMSNorm gains, loaded into registers ahead of use so that their loads
-// overlap the exchange that delivers x (elements 4j..4j+3 for j = tid + 224k).
-struct Gains {
-  float4 v[4];
-  __device__ __forceinline__ void load(const float* g, int n) {
-    const float4* g4 = reinterpret_cast<const float4*>(g);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const int j = threadIdx.x + k * kConsumerThreads;
-      if (j < (n >> 2)) v[k] = __ldg(g4 + j);
-    }
-  }
-};
-
-// out = RMSNorm(x, g) (paper §11.2: ss/n + eps, 1/sqrt, then (x*g)*r), given
-// ss = this thread's share of the sum of x^2 and the preloaded gains.
-__device__ inline void rmsnorm_finish(float* out, const float* x, const Gains& gp, const float* g,
-                                      int n, float eps, float ss, float* red) {
-  const float tot = block_sum(ss, red);  // its barriers also publish x
-  const float r = 1.0f / sqrtf(tot / (float)n + eps);
-  const int n4 = n >> 2;
-  const float4* x4 = reinterpret_cast<const float4*>(x);
-  float4* o4 = reinterpret_cast<float4*>(out);
-  auto emit = [&](int j, const float4& gv) {
-    const float4 xv = x4[j];
-    o4[j] = make_float4((xv.x * gv.x) * r, (xv.y * gv.y) * r, (xv.z * gv.z) * r,
-                        (xv.w * gv.w) * r);
-  };
-#pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    const int j = threadIdx.x + k * kConsumerThreads;
-    if (j < n4) emit(j, gp.v[k]);
-  }
-  for (int j = threadIdx.x + 4 * kConsumerThreads; j < n4; j += kConsumerThreads)
-    emit(j, __ldg(reinterpret_cast<const float4*>(g) + j));
-  named_bar_sync(kBarConsumers, kConsumerThreads);
-}
-
-// RMSNorm of kB vectors (x_b at x + b * n, out_b at out + b * vs) with the
-// same gains; ss[b] = this thread's share of sum x_b^2.
-template <int kB>
-__device__ inline void rmsnorm_finish_n(float* out, int vs, const float* x, const Gains& gp,
-                                        const float* g, int n, float eps, float (&ss)[kB],
-                                        float* red) {
-  if constexpr (kB == 1) {
-    rmsnorm_finish(out, x, gp, g, n, eps, ss[0], red);
-    return;
-  }
-  block_sum_n<kB>(ss, red);  // its barriers also publish x
-  const int n4 = n >> 2;
-#pragma unroll
-  for (int b = 0; b < kB; ++b) {
-    const float r = 1.0f / sqrtf(ss[b] / (float)n + eps);
-    const float4* x4 = reinterpret_cast<const float4*>(x + (size_t)b * n);
-    float4* o4 = reinterpret_cast<float4*>(out + (size_t)b * vs);
-    auto emit = [&](int j, const float4& gv) {
-      const float4 xv = x4[j];
-      o4[j] = make_float4((xv.x * gv.x) * r, (xv.y * gv.y) * r, (xv.z * gv.z) * r,
-                          (xv.w * gv.w) * r);
-    };
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const int j = threadIdx.x + k * kConsumerThreads;
-      if (j < n4) emit(j, gp.v[k]);
-    }
-    for (int j = threadIdx.x + 4 * kConsumerThreads; j < n4; j += kConsumerThreads)
-      emit(j, __ldg(reinterpret_cast<const float4*>(g) + j));
-  }
-  named_bar_sync(kBarConsumers, kConsumerThreads);
-}
-
-// This thread's share of sum x^2 when no exchange delivered x.
-__device__ inline float sum_sq(const float* x, int n) {
-  float ss = 0.f;
-  for (int j = threadIdx.x; j < n; j += kConsumerThreads) ss = fmaf(x[j], x[j], ss);
-  return ss;
+  for (int i = 1; i < kMaxBatch; ++i)
+    if (b == i) v = sc[i];
+  return v;
 }
 
 // Publishes GEMV rows as tagged words (M words per sequence). With swiglu
@@ -405,14 +368,18 @@ struct EpiTag {
   unsigned tag;
   int M;
   bool swiglu;
+  float scale[kMaxBatch];
   __device__ __forceinline__ void store(int row, float v) { store_b(row, 0, v); }
   __device__ __forceinline__ void store_b(int row, int b, float v) {
-    st_tag(out + (size_t)b * M + row, tag, v);
+    st_tag(out + (size_t)b * M + row, tag, v * pick_scale(scale, b));
   }
   __device__ __forceinline__ void store_pair(int row, float v0, float v1) {
     store_pair_b(row, 0, v0, v1);
   }
   __device__ __forceinline__ void store_pair_b(int row, int b, float v0, float v1) {
+    const float sc = pick_scale(scale, b);
+    v0 *= sc;
+    v1 *= sc;
     if (swiglu) {
       st_tag(out + (size_t)b * M + (row >> 1), tag, (v0 / (1.0f + expf(-v0))) * v1);
     } else {
@@ -428,6 +395,7 @@ template <int kB>
 struct EpiArgmax {
   float* out;
   int V;
+  float scale[kMaxBatch];  // RMSNorm factor of sequence b's input
   float bv[kB];
   int bi[kB];
   __device__ __forceinline__ void init() {
@@ -444,6 +412,7 @@ struct EpiArgmax {
     store_b(row + 1, b, v1);
   }
   __device__ __forceinline__ void store_b(int row, int b, float v) {
+    v *= pick_scale(scale, b);
     out[(size_t)b * V + row] = v;
 #pragma unroll
     for (int bb = 0; bb < kB; ++bb)
@@ -819,19 +788,62 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
   int token[kB];
 #pragma unroll
   for (int b = 0; b < kB; ++b) token[b] = a.start_tokens[b];
-  // x += (published vector), identically in every CTA; ss[b] += the new x_b^2
-  auto add_published = [&](const unsigned long long* src, unsigned tag, float(&ss)[kB]) {
-    const int hp = a.d >> 1;
-    const bool ok = poll_pairs<kPollDepth>(src, kB * hp, tag, pc, [&](int p, float v0, float v1) {
-      const float x0 = xs[2 * p] + v0, x1 = xs[2 * p + 1] + v1;
-      xs[2 * p] = x0;
-      xs[2 * p + 1] = x1;
-      const int pb = kB == 1 ? 0 : p / hp;
+  const int n4 = a.d >> 2;  // quads of a residual vector
+  // The RMSNorm of a phase input, paper §11.2: x_b = (x * g) * r with r =
+  // 1/sqrt(ss/n + eps). The thread that owns quad j of x (j = tid + 224 k over
+  // the kB stacked vectors) writes vec = x * g for it and adds x^2 to its share
+  // ss[b]; r goes to the GEMV epilogue (EpiTag, EpiArgmax scale), so no pass
+  // over the vector and no block reduction stand between the exchange and the
+  // GEMV.
+  auto norm_quad = [&](int j, const float4& x, const float4& g, float(&ss)[kB]) {
+    const int pb = kB == 1 ? 0 : j / n4, jj = j - pb * n4;
+    reinterpret_cast<float4*>(vec + (size_t)pb * vs)[jj] =
+        make_float4(x.x * g.x, x.y * g.y, x.z * g.z, x.w * g.w);
 #pragma unroll
-      for (int b = 0; b < kB; ++b)
-        if (b == pb) ss[b] = fmaf(x1, x1, fmaf(x0, x0, ss[b]));
+    for (int b = 0; b < kB; ++b)
+      if (b == pb) ss[b] = fmaf(x.w, x.w, fmaf(x.z, x.z, fmaf(x.y, x.y, fmaf(x.x, x.x, ss[b]))));
+  };
+  // x += (published vector), identically in every CTA, and the norm input
+  auto add_published = [&](const unsigned long long* src, unsigned tag, const float* gain,
+                           float(&ss)[kB]) {
+    const float4* g4 = reinterpret_cast<const float4*>(gain);
+    return poll_quads<2>(src, kB * n4, tag, g4, n4, pc, [&](int j, float4 v, const float4& g) {
+      float4* x4 = reinterpret_cast<float4*>(xs) + j;
+      float4 x = *x4;
+      x.x += v.x;
+      x.y += v.y;
+      x.z += v.z;
+      x.w += v.w;
+      *x4 = x;
+      norm_quad(j, x, g, ss);
     });
-    return vote_ok(ok, s_abort);
+  };
+  // the norm input when no exchange delivered x (the embedding row)
+  auto norm_local = [&](const float* gain, float(&ss)[kB]) {
+    const float4* g4 = reinterpret_cast<const float4*>(gain);
+    for (int j = tid; j < kB * n4; j += kConsumerThreads)
+      norm_quad(j, reinterpret_cast<const float4*>(xs)[j], __ldg(g4 + j % n4), ss);
+  };
+  // r_b from every thread's share of ss_b: warp sums go to red, and the block
+  // vote that follows the exchange publishes them (and x, vec)
+  auto norm_scales = [&](bool ok, float(&ss)[kB], float(&rs)[kMaxBatch]) {
+    const int warp = tid >> 5, lane = tid & 31;
+#pragma unroll
+    for (int b = 0; b < kB; ++b) {
+      const float t = warp_sum(ss[b]);
+      if (lane == 0) red[warp * kB + b] = t;
+    }
+    if (!vote_ok(ok, s_abort)) return false;
+#pragma unroll
+    for (int b = 0; b < kMaxBatch; ++b) {
+      float t = 0.f;
+      if (b < kB) {
+#pragma unroll
+        for (int w = 0; w < kConsumerWarps; ++w) t += red[w * kB + b];
+      }
+      rs[b] = b < kB ? 1.0f / sqrtf(t / (float)a.d + a.eps) : 1.0f;
+    }
+    return true;
   };
   for (int s = 0; s < a.n_steps; ++s) {
     const int pos = a.start_pos + s;
@@ -879,23 +891,24 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
 #pragma unroll 1
       for (int k = 0; k < 4; ++k) {
         if (k == 0) att_prefetch_l2<kB>(a, l, pos);
+        if (k == 1 && !attention_phase<kB>(a, l, pos, el, el + 1, asm_, red, pc)) return false;
+        const StagePlan plan = plans[k];
+        float rs[kMaxBatch];
+#pragma unroll
+        for (int b = 0; b < kMaxBatch; ++b) rs[b] = 1.0f;
         if (k == 0 || k == 2) {
-          // x += (the previous phase's published output), then x_b = RMSNorm(x, g)
+          // x += (the previous phase's published output); the input is x * g,
+          // scaled by r in the epilogue
           const float* gain = reinterpret_cast<const float*>(lw + (k == 0 ? a.o_gatt : a.o_gffn));
-          Gains gp;
-          gp.load(gain, a.d);
           float ss[kB];
 #pragma unroll
           for (int b = 0; b < kB; ++b) ss[b] = 0.f;
-          if (k == 2 || l > 0) {
-            if (!add_published(k == 0 ? a.x_f : a.x_o, k == 0 ? el - 1 : el + 2, ss)) return false;
-          } else {
-#pragma unroll
-            for (int b = 0; b < kB; ++b) ss[b] = sum_sq(xs + (size_t)b * a.d, a.d);
-          }
-          rmsnorm_finish_n<kB>(vec, vs, xs, gp, gain, a.d, a.eps, ss, red);
+          bool ok = true;
+          if (k == 2 || l > 0) ok = add_published(k == 0 ? a.x_f : a.x_o, k == 0 ? el - 1 : el + 2,
+                                                  gain, ss);
+          else norm_local(gain, ss);
+          if (!norm_scales(ok, ss, rs)) return false;
         } else if (k == 1) {
-          if (!attention_phase<kB>(a, l, pos, el, el + 1, asm_, red, pc)) return false;
           const int hp = a.d >> 1;
           const bool ok = poll_pairs<kPollDepth>(a.x_attn, kB * hp, el + 1, pc,
                                                  [&](int p, float v0, float v1) {
@@ -921,9 +934,9 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
         // partials take el + 1)
         const int M = k == 0 ? a.d + 2 * a.kvd : k == 2 ? 2 * a.F : a.d;
         const int K = k == 3 ? a.F : a.d;
-        const StagePlan plan = plans[k];
         unsigned long long* out = k == 0 ? a.x_qkv : k == 1 ? a.x_o : k == 2 ? a.x_h13 : a.x_f;
-        EpiTag e{out, el + (k == 0 ? 0u : (unsigned)k + 1u), k == 2 ? a.F : M, k == 2};
+        EpiTag e{out, el + (k == 0 ? 0u : (unsigned)k + 1u), k == 2 ? a.F : M, k == 2,
+                 {rs[0], rs[1], rs[2], rs[3]}};
         if constexpr (kQ8) {
           if (!consume_phase<false, kQ8>(r, g, plan, vec, 1, K, seg, e, a.err, a.err_host,
                                          s_abort))
@@ -934,21 +947,17 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
         }
       }
     }
+    float rs[kMaxBatch];
     {
-      Gains gp;
-      gp.load(a.g_final, a.d);
       float ss[kB];
 #pragma unroll
       for (int b = 0; b < kB; ++b) ss[b] = 0.f;
-      if (a.L > 0) {
-        if (!add_published(a.x_f, es + per_step - 2, ss)) return false;
-      } else {
-#pragma unroll
-        for (int b = 0; b < kB; ++b) ss[b] = sum_sq(xs + (size_t)b * a.d, a.d);
-      }
-      rmsnorm_finish_n<kB>(vec, vs, xs, gp, a.g_final, a.d, a.eps, ss, red);
+      bool ok = true;
+      if (a.L > 0) ok = add_published(a.x_f, es + per_step - 2, a.g_final, ss);
+      else norm_local(a.g_final, ss);
+      if (!norm_scales(ok, ss, rs)) return false;
     }
-    EpiArgmax<kB> ea{a.logits, a.V};
+    EpiArgmax<kB> ea{a.logits, a.V, {rs[0], rs[1], rs[2], rs[3]}};
     ea.init();
     if constexpr (kQ8) {
       if (!consume_phase<false, kQ8>(r, g, plans[4], vec, 1, a.d, seg, ea, a.err, a.err_host,
