@@ -73,6 +73,8 @@ def lib():
                                         ctypes.c_int, ctypes.POINTER(ctypes.c_int)]
         L.orc_quantize_rows_q8.restype = None
         L.orc_quantize_rows_q8.argtypes = [P, i64, i64, P, P]
+        L.orc_quantize_rows_q4.restype = None
+        L.orc_quantize_rows_q4.argtypes = [P, i64, i64, P, P]
         L.orc_gemv_q8_f64.restype = None
         L.orc_gemv_q8_f64.argtypes = [P, P, P, P, i64, i64]
         L.orc_forward.restype = ctypes.c_int
@@ -128,8 +130,19 @@ def quantize_rows_q8(W: np.ndarray):
     return q, s
 
 
+def quantize_rows_q4(W: np.ndarray):
+    """4-bit codes (one per int8, in [-7, 7]) and row scales of W float32 [M, K]
+    (see orc_quantize_rows_q4)."""
+    W = np.ascontiguousarray(W, dtype=np.float32)
+    M, K = W.shape
+    q = np.empty((M, K), dtype=np.int8)
+    s = np.empty(M, dtype=np.float32)
+    lib().orc_quantize_rows_q4(_ptr(W), M, K, _ptr(q), _ptr(s))
+    return q, s
+
+
 def gemv_q8(q: np.ndarray, s: np.ndarray, x: np.ndarray) -> np.ndarray:
-    """y = (s_i q_ij) x in double."""
+    """y = (s_i q_ij) x in double (the codes of quantize_rows_q8 or _q4)."""
     q = np.ascontiguousarray(q, dtype=np.int8)
     s = np.ascontiguousarray(s, dtype=np.float32)
     x = np.ascontiguousarray(x, dtype=np.float64)

@@ -103,29 +103,34 @@ void gemv(const float* W, const Acc* x, Acc* y, int64_t M, int64_t K) {
   }
 }
 
-// Weight-only 8-bit codes, one float32 scale per output row. Every decision
+// Weight-only codes with qmax levels on each side of zero (127 for 8-bit
+// codes, 7 for 4-bit ones), one float32 scale per output row. Every decision
 // is taken in float32, so that any implementation of the same definition
-// finds the same codes: a_r = max_j |W_rj|; s_r = a_r / 127; q_rj = the
-// integer nearest to W_rj / s_r (ties to even), which lies in [-127, 127];
+// finds the same codes: a_r = max_j |W_rj|; s_r = a_r / qmax; q_rj = the
+// integer nearest to W_rj / s_r (ties to even), which lies in [-qmax, qmax];
 // an all-zero row has s_r = 0 and codes 0. The weight a code stands for is
 // s_r * q_rj.
-void quantize_rows(const float* W, int64_t M, int64_t K, int8_t* q, float* s) {
+void quantize_rows_levels(const float* W, int64_t M, int64_t K, float qmax, int8_t* q, float* s) {
   for (int64_t i = 0; i < M; ++i) {
     const float* w = W + i * K;
     float a = 0.0f;
     for (int64_t j = 0; j < K; ++j) a = std::fmax(a, std::fabs(w[j]));
-    const float sc = a / 127.0f;
+    const float sc = a / qmax;
     s[i] = sc;
     for (int64_t j = 0; j < K; ++j) {
       float c = 0.0f;
       if (sc != 0.0f) {
         c = std::nearbyint(w[j] / sc);  // default rounding: nearest, ties to even
-        if (c > 127.0f) c = 127.0f;
-        if (c < -127.0f) c = -127.0f;
+        if (c > qmax) c = qmax;
+        if (c < -qmax) c = -qmax;
       }
       q[i * K + j] = (int8_t)c;
     }
   }
+}
+
+void quantize_rows(const float* W, int64_t M, int64_t K, int8_t* q, float* s) {
+  quantize_rows_levels(W, M, K, 127.0f, q, s);
 }
 
 // y[i] = sum_j (s_i q_ij) x[j]: the GEMV of the weights the codes stand for.
@@ -432,6 +437,10 @@ void orc_quantize_rows_q8(const float* W, int64_t M, int64_t K, int8_t* q, float
 void orc_gemv_q8_f64(const int8_t* q, const float* s, const double* x, double* y, int64_t M,
                      int64_t K) {
   gemv_q8<double>(q, s, x, y, M, K);
+}
+
+void orc_quantize_rows_q4(const float* W, int64_t M, int64_t K, int8_t* q, float* s) {
+  quantize_rows_levels(W, M, K, 7.0f, q, s);
 }
 
 void orc_gemv_f64(const float* W, const double* x, double* y, int64_t M, int64_t K) {

@@ -58,7 +58,12 @@ void orc_model_free(void* model);
  * q[i][j] = nearest integer (ties to even) to W[i][j] / s[i], all in float32
  * (0 codes and scale for an all-zero row). */
 void orc_quantize_rows_q8(const float* W, int64_t M, int64_t K, int8_t* q, float* s);
-/* y[i] = sum_j (s[i] * q[i][j]) * x[j] in double. */
+/* Weight-only 4-bit codes (quantization future work, read as symmetric
+ * per-row codes like the 8-bit ones): s[i] = max_j |W[i][j]| / 7 and q[i][j]
+ * = nearest integer (ties to even) to W[i][j] / s[i], in [-7, 7], all in
+ * float32; one code per int8 (the packing is the GPU format's business). */
+void orc_quantize_rows_q4(const float* W, int64_t M, int64_t K, int8_t* q, float* s);
+/* y[i] = sum_j (s[i] * q[i][j]) * x[j] in double (8-bit or 4-bit codes). */
 void orc_gemv_q8_f64(const int8_t* q, const float* s, const double* x, double* y, int64_t M,
                      int64_t K);
 void orc_gemv_f64(const float* W, const double* x, double* y, int64_t M, int64_t K);

@@ -376,6 +376,49 @@ def test_q8_gemv_is_the_gemv_of_the_weights_the_codes_stand_for():
                        x * 127 * float(np.float32(1 / 127)), rtol=0, atol=1e-15)
 
 
+# ---- weight-only 4-bit codes (the same definition with 7 levels on each side
+# of zero: s = max|w| / 7, q = nearest(w / s), ties to even, in [-7, 7]) ----
+
+def test_q4_integer_rows_with_max_7_keep_their_values_and_round_ties_to_even():
+    W = np.array([[7, 0.5, 1.5, 2.5, -0.5, -1.5, 3.5, -2.5, -7, 4, 6.5, -5.5]], np.float32)
+    q, s = oracle.quantize_rows_q4(W)
+    assert s[0] == np.float32(1.0)
+    assert q.tolist() == [[7, 0, 2, 2, 0, -2, 4, -2, -7, 4, 6, -6]]
+
+
+def test_q4_codes_reach_7_at_the_row_maximum_and_stay_within_half_a_step():
+    W = (RNG.standard_normal((40, 256)) * 0.02).astype(np.float32)
+    q, s = oracle.quantize_rows_q4(W)
+    assert np.abs(q).max() == 7
+    for i in range(40):
+        j = int(np.argmax(np.abs(W[i])))
+        assert abs(int(q[i, j])) == 7
+        err = np.abs(W[i].astype(np.float64) - float(s[i]) * q[i].astype(np.float64))
+        assert err.max() <= 0.5 * float(s[i]) * (1 + 1e-6)  # nearest level, float32 division
+    assert float(s[0]) == float(np.float32(np.abs(W[0]).max()) / np.float32(7.0))
+
+
+def test_q4_zero_row_sign_symmetry_and_power_of_two_scaling():
+    W = RNG.standard_normal((9, 64)).astype(np.float32)
+    W[4] = 0.0
+    q, s = oracle.quantize_rows_q4(W)
+    assert s[4] == 0.0 and not q[4].any()
+    qn, sn = oracle.quantize_rows_q4(-W)
+    assert np.array_equal(qn, -q) and np.array_equal(sn, s)
+    q2, s2 = oracle.quantize_rows_q4(W * np.float32(8.0))  # exact in float32
+    assert np.array_equal(q2, q) and np.array_equal(s2, s * np.float32(8.0))
+
+
+def test_q4_code_is_the_nearest_of_the_15_levels_by_brute_force():
+    W = (RNG.standard_normal((6, 50)) * 0.02).astype(np.float32)
+    q, s = oracle.quantize_rows_q4(W)
+    for i in range(6):
+        levels = np.arange(-7, 8, dtype=np.float64) * float(s[i])
+        for j in range(50):
+            d = np.abs(levels - float(W[i, j]))
+            assert d[int(q[i, j]) + 7] <= d.min() * (1 + 1e-6) + 1e-15
+
+
 def _representable_blob(cfg, seed):
     """A blob whose every weight matrix row is k * 2^-12 with integer |k| <= 127
     and some |k| == 127: its 8-bit codes and scales are exact."""
