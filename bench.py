@@ -50,8 +50,9 @@ def parse():
     ap.add_argument("--warmup", type=int, default=256)
     ap.add_argument("--impl", default="tvl", choices=["tvl", "reference"])
     ap.add_argument("--workload", default="110m", choices=["110m", "110m-long", "tiny", "7b"])
-    ap.add_argument("--weights", default="f32", choices=["f32", "q8"],
-                    help="q8: weight-only 8-bit rows (tvl_config.weight_bits = 8)")
+    ap.add_argument("--weights", default="f32", choices=["f32", "q8", "q4"],
+                    help="q8: weight-only 8-bit rows (tvl_config.weight_bits = 8); "
+                         "q4: weight-only 4-bit rows (--gemv-sweep only)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
@@ -285,18 +286,19 @@ def gemv_sweep(args):
     out = []
     for i, (M, K) in enumerate(synth.GEMV_SHAPES):
         W, x = synth.gemv_operands(M, K, i)
-        q8 = args.weights == "q8"
-        wbytes = tvl.tvl_q8_bytes(M, K) if q8 else 4 * M * K
+        packed = {"q8": (tvl.tvl_q8_bytes, tvl.tvl_quantize_q8, tvl.tvl_gemv_q8),
+                  "q4": (tvl.tvl_q4_bytes, tvl.tvl_quantize_q4, tvl.tvl_gemv_q4)}.get(args.weights)
+        wbytes = packed[0](M, K) if packed else 4 * M * K
         nbytes = wbytes + 4 * (M + K)
         copies = max(1, math.ceil(3 * l2 / wbytes))
-        if q8:  # packed 8-bit rows of W, one copy per rotation slot
+        if packed:  # packed 8-bit or 4-bit rows of W, one copy per rotation slot
             dW1 = torch.from_numpy(W).cuda()
             dW = torch.empty((copies, wbytes), dtype=torch.uint8, device="cuda")
             for c in range(copies):
-                tvl.tvl_quantize_q8(dW1.data_ptr(), dW[c].data_ptr(), M, K)
+                packed[1](dW1.data_ptr(), dW[c].data_ptr(), M, K)
             torch.cuda.synchronize()
             del dW1
-            call = tvl.tvl_gemv_q8
+            call = packed[2]
         else:
             dW = torch.from_numpy(W).cuda().repeat(copies, 1).reshape(copies, M, K)
             call = tvl.tvl_gemv
@@ -330,6 +332,10 @@ def gemv_sweep(args):
 
 def main():
     args = parse()
+    if args.weights == "q4" and not args.gemv_sweep:
+        print(json.dumps({"error": "--weights q4 is for --gemv-sweep: models decode with "
+                                   "float32 or 8-bit rows"}))
+        return 2
     rank, local_rank, world = dist_env()
     from paper_2601_03324_gb300 import synth
     cfg = synth.model_config("110m" if args.workload == "110m-long" else args.workload)

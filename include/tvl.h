@@ -53,7 +53,8 @@ typedef struct {
   int32_t weight_bits;  /* 0: float32 weights as in the blob; 8: tvl_load turns every weight
                            matrix (and the embedding table) into 8-bit rows, as
                            tvl_quantize_q8 defines, and decodes with them; dim and
-                           hidden_dim must then be multiples of 16 */
+                           hidden_dim must then be multiples of 16. Any other value is
+                           TVL_E_INVAL (4-bit rows serve the standalone tvl_gemv_q4 only) */
   int32_t max_batch;    /* sequences one launch may decode together, 0 or 1 (one) to 4;
                            each sequence slot gets its own KV cache and exchange buffers.
                            More than one needs weight_bits 0 */
@@ -188,6 +189,32 @@ tvl_status tvl_quantize_q8(const float* W, void* Wq8, int32_t rows, int32_t cols
  * TVL_E_INVAL / TVL_E_UNSUPPORTED. Queued on `stream`, does not wait,
  * allocates nothing. */
 tvl_status tvl_gemv_q8(const void* Wq8, const float* x, float* y, int32_t d_out, int32_t d_in,
+                       void* stream);
+
+/* Weight-only 4-bit rows: the same reading of the paper's quantization
+ * future work (§ Future Work: Quantization names 4-bit weights unpacked on
+ * the fly) with 7 levels on each side of zero. A matrix W [rows x cols]
+ * becomes packed rows of 16 + cols/2 bytes: the float32 scale
+ * s = max_j |W[r][j]| / 7 (bytes 0-3), twelve zero bytes, then the codes
+ * q[r][j] = the integer nearest to W[r][j] / s (ties to even, in [-7, 7]; an
+ * all-zero row has s = 0 and codes 0), every step in float32, two per byte as
+ * 4-bit two's complement: byte m holds column 2m in its low nibble and column
+ * 2m + 1 in its high nibble. The code stands for the weight s * q. cols must
+ * be a positive multiple of 32. tvl_q4_bytes: bytes of the packed rows (0 if
+ * rows < 1 or cols is invalid). */
+size_t tvl_q4_bytes(int32_t rows, int32_t cols);
+
+/* Quantize W (device, float32, row-major, 16-byte aligned) into Wq4 (device,
+ * tvl_q4_bytes(rows, cols) bytes, 16-byte aligned), on `stream`, without
+ * waiting. Errors: TVL_E_INVAL (null pointer, bad size), TVL_E_ALIGN. */
+tvl_status tvl_quantize_q4(const float* W, void* Wq4, int32_t rows, int32_t cols, void* stream);
+
+/* y = W' x for the weights W' the packed 4-bit rows stand for (y[r] = s_r *
+ * sum_j q[r][j] x[j]); Wq4 and x device pointers, 16-byte aligned; d_in a
+ * multiple of 32 and at most 32736 (a packed row fits one 16 KB stage), else
+ * TVL_E_INVAL / TVL_E_ALIGN / TVL_E_UNSUPPORTED. Queued on `stream`, does not
+ * wait, allocates nothing. Models decode with float32 or 8-bit rows only. */
+tvl_status tvl_gemv_q4(const void* Wq4, const float* x, float* y, int32_t d_out, int32_t d_in,
                        void* stream);
 
 /* tvl_gemv without any allocation. The paper has no counterpart: this entry

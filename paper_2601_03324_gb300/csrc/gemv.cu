@@ -57,7 +57,7 @@ struct GemvSched {
   }
 };
 
-template <bool kQ8>
+template <bool kQ8, bool kQ4 = false>
 __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_constant__ GemvArgs a) {
   extern __shared__ __align__(128) unsigned char smem[];
   Ring r;
@@ -94,7 +94,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   named_bar_sync(kBarConsumers, kConsumerThreads);
   if (a.S == 1) {
     EpiStore e{a.y};
-    consume_phase<true, kQ8>(r, g, p, xs, 1, a.Kc, seg, e, nullptr, nullptr, s_abort);
+    consume_phase<true, kQ8, kQ4>(r, g, p, xs, 1, a.Kc, seg, e, nullptr, nullptr, s_abort);
     return;
   }
   EpiPart e{a.part};
@@ -164,6 +164,41 @@ __global__ void quantize_q8_kernel(const float* __restrict__ W, unsigned char* _
     const float4 v = w4[e];
     codes[e] = (code(v.x) & 0xff) | ((code(v.y) & 0xff) << 8) | ((code(v.z) & 0xff) << 16) |
                (code(v.w) << 24);
+  }
+}
+
+// 4-bit codes of W [M x K] as packed rows (16 + K/2 bytes: scale, 12 zero
+// bytes, two codes per byte with the even column in the low nibble), one warp
+// per row; lane takes code word e (columns 8e..8e+7). The same float32
+// decisions as the 8-bit codes with 7 levels: s = max|w| / 7, code = nearest
+// integer to w / s, ties to even, in [-7, 7]. Requires K % 32 == 0.
+__global__ void quantize_q4_kernel(const float* __restrict__ W, unsigned char* __restrict__ Q,
+                                   int M, int K) {
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (row >= M) return;
+  const float4* w4 = reinterpret_cast<const float4*>(W + (size_t)row * K);
+  const int n4 = K >> 2, nw = K >> 3;
+  float amax = 0.f;
+  for (int e = lane; e < n4; e += 32) {
+    const float4 v = w4[e];
+    amax = fmaxf(amax, fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w))));
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
+  const float sc = __fdiv_rn(amax, 7.0f);
+  unsigned char* out = Q + (size_t)row * (16 + K / 2);
+  if (lane < 4) reinterpret_cast<unsigned*>(out)[lane] = lane == 0 ? __float_as_uint(sc) : 0u;
+  unsigned* words = reinterpret_cast<unsigned*>(out + 16);
+  auto code = [&](float v) -> unsigned {
+    if (sc == 0.f) return 0u;
+    int c = __float2int_rn(__fdiv_rn(v, sc));
+    c = c > 7 ? 7 : (c < -7 ? -7 : c);
+    return (unsigned)c & 0xFu;
+  };
+  for (int e = lane; e < nw; e += 32) {
+    const float4 a = w4[2 * e], b = w4[2 * e + 1];
+    words[e] = code(a.x) | (code(a.y) << 4) | (code(a.z) << 8) | (code(a.w) << 12) |
+               (code(b.x) << 16) | (code(b.y) << 20) | (code(b.z) << 24) | (code(b.w) << 28);
   }
 }
 
@@ -478,6 +513,83 @@ extern "C" tvl_status tvl_gemv_q8(const void* Wq8, const float* x, float* y, int
   TVL_CK(cudaFuncSetAttribute((const void*)gemv_stream_kernel<true>,
                               cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
   gemv_stream_kernel<true><<<G, kThreads, smem, s>>>(a);
+  TVL_CK(cudaGetLastError());
+  return TVL_OK;
+}
+
+// ---- weight-only 4-bit rows: quantization and GEMV ---------------------------------
+
+extern "C" size_t tvl_q4_bytes(int32_t rows, int32_t cols) {
+  if (rows < 1 || cols < 32 || cols % 32 != 0) return 0;
+  return (size_t)rows * (size_t)(16 + cols / 2);
+}
+
+extern "C" tvl_status tvl_quantize_q4(const float* W, void* Wq4, int32_t rows, int32_t cols,
+                                      void* stream) {
+  if (!W || !Wq4 || tvl_q4_bytes(rows, cols) == 0) {
+    set_error("tvl_quantize_q4: null pointer, or cols not a positive multiple of 32");
+    return TVL_E_INVAL;
+  }
+  if ((uintptr_t)W % 16 || (uintptr_t)Wq4 % 16) {
+    set_error("tvl_quantize_q4: W and Wq4 must be 16-byte aligned");
+    return TVL_E_ALIGN;
+  }
+  const int threads = 256, rows_per_block = threads / 32;
+  quantize_q4_kernel<<<(rows + rows_per_block - 1) / rows_per_block, threads, 0,
+                       (cudaStream_t)stream>>>(W, (unsigned char*)Wq4, rows, cols);
+  TVL_CK(cudaGetLastError());
+  return TVL_OK;
+}
+
+extern "C" tvl_status tvl_gemv_q4(const void* Wq4, const float* x, float* y, int32_t d_out,
+                                  int32_t d_in, void* stream) {
+  if (!Wq4 || !x || !y || tvl_q4_bytes(d_out, d_in) == 0) {
+    set_error("tvl_gemv_q4: null pointer, or d_in not a positive multiple of 32");
+    return TVL_E_INVAL;
+  }
+  if ((uintptr_t)Wq4 % 16 || (uintptr_t)x % 16) {
+    set_error("tvl_gemv_q4: Wq4 and x must be 16-byte aligned");
+    return TVL_E_ALIGN;
+  }
+  const int Kw = 4 + d_in / 8;  // words per packed row
+  if (Kw > kStageFloats) {
+    set_error("tvl_gemv_q4: a packed row must fit one 16 KB stage (d_in <= 32736)");
+    return TVL_E_UNSUPPORTED;
+  }
+  cudaStream_t s = (cudaStream_t)stream;
+  int dev = 0, sms = 0, max_optin = 0;
+  TVL_CK(cudaGetDevice(&dev));
+  TVL_CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  TVL_CK(cudaDeviceGetAttribute(&max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev));
+  GemvArgs a{};
+  a.W = reinterpret_cast<const float*>(Wq4);
+  a.x = x;
+  a.y = y;
+  a.M = d_out;
+  a.K = d_in;
+  a.S = 1;
+  a.Kc = Kw;
+  a.nv = d_out;
+  const int G = d_out < sms ? d_out : sms;
+  const int xbytes = (int)a128(4LL * d_in), segb = (int)a128(kMaxSegParts * 4);
+  const int bars = (int)a128(kRingBarBytes);
+  const int misc = 128;
+  int nst = (max_optin - xbytes - segb - bars - misc) / kStageBytes;
+  if (nst > kMaxStages) nst = kMaxStages;
+  if (nst < 2) {
+    set_error("tvl_gemv_q4: not enough shared memory");
+    return TVL_E_UNSUPPORTED;
+  }
+  a.nst = nst;
+  a.sm_ring = 0;
+  a.sm_bars = nst * kStageBytes;
+  a.sm_x = a.sm_bars + bars;
+  a.sm_seg = a.sm_x + xbytes;
+  a.sm_misc = a.sm_seg + segb;
+  const int smem = a.sm_misc + misc;
+  TVL_CK(cudaFuncSetAttribute((const void*)gemv_stream_kernel<false, true>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+  gemv_stream_kernel<false, true><<<G, kThreads, smem, s>>>(a);
   TVL_CK(cudaGetLastError());
   return TVL_OK;
 }

@@ -340,6 +340,48 @@ __device__ __forceinline__ float row_partial_q8(const int* c0, const float4* x4,
   return (a.x + a.y) + (a.z + a.w);
 }
 
+// 4-bit weight rows: a packed row is 16 + K/2 bytes (the float32 scale, 12
+// zero bytes, then two codes per byte, low nibble first, each a 4-bit two's
+// complement integer in [-7, 7]); in a stage a row is 4 + K/8 words. Code
+// word e holds codes 8e..8e+7 and meets x float4 2e and 2e + 1.
+__device__ __forceinline__ void fma_nibbles(float4& acc, int w, const float4& xa,
+                                            const float4& xb) {
+  // code + 8 (in [1, 15]) as the low bits of the float 2^23 + (code + 8):
+  // a shift, a mask and an OR per code, then one exact subtraction
+  const unsigned u = (unsigned)w ^ 0x88888888u;
+  auto c = [u](int k) {
+    return __uint_as_float(0x4B000000u | ((u >> (4 * k)) & 0xFu)) - 8388616.0f;
+  };
+  acc.x = fmaf(c(0), xa.x, acc.x);
+  acc.y = fmaf(c(1), xa.y, acc.y);
+  acc.z = fmaf(c(2), xa.z, acc.z);
+  acc.w = fmaf(c(3), xa.w, acc.w);
+  acc.x = fmaf(c(4), xb.x, acc.x);
+  acc.y = fmaf(c(5), xb.y, acc.y);
+  acc.z = fmaf(c(6), xb.z, acc.z);
+  acc.w = fmaf(c(7), xb.w, acc.w);
+}
+
+// Lane partials of sum_j q_j x_j for two 4-bit rows sharing x (nw code words).
+__device__ __forceinline__ float2 row2_partial_q4(const int* c0, const int* c1, const float4* x4,
+                                                  int nw, int lane) {
+  float4 a = make_float4(0.f, 0.f, 0.f, 0.f), b = a;
+#pragma unroll 4
+  for (int e = lane; e < nw; e += 32) {
+    const float4 xa = x4[2 * e], xb = x4[2 * e + 1];
+    fma_nibbles(a, c0[e], xa, xb);
+    fma_nibbles(b, c1[e], xa, xb);
+  }
+  return make_float2((a.x + a.y) + (a.z + a.w), (b.x + b.y) + (b.z + b.w));
+}
+
+__device__ __forceinline__ float row_partial_q4(const int* c0, const float4* x4, int nw, int lane) {
+  float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+  for (int e = lane; e < nw; e += 32) fma_nibbles(a, c0[e], x4[2 * e], x4[2 * e + 1]);
+  return (a.x + a.y) + (a.z + a.w);
+}
+
 // Warp-level bounded wait for stage gs in `slot` (all lanes poll, lane 0
 // applies the limit): first until the producer has queued that stage into the
 // slot, then until its bytes have landed. Returns the same answer in every
@@ -406,14 +448,14 @@ __device__ inline bool warp_wait_full(const Ring& r, int slot, uint32_t gs, int*
 // (deferred rows) from the thread that adds the rows' partials at the end of
 // the phase. seg is shared scratch for those partials. Ends with a barrier of the consumer
 // warps; returns false on abort, identically in every consumer thread.
-template <bool kXReg = true, bool kQ8 = false, class Epi>
+template <bool kXReg = true, bool kQ8 = false, bool kQ4 = false, class Epi>
 __device__ inline bool consume_phase(const Ring& r, uint32_t& g, const StagePlan& p,
                                      const float* xs, int S, int Kc, float* seg, Epi& epi,
                                      int* err, int* err_host, volatile int* s_abort) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // Rows of at most 1024 floats (whole rows in a stage, one K-chunk): each lane
   // keeps its x slice in registers for the whole phase.
-  const bool xreg = kXReg && !kQ8 && (p.spr == 1) && (p.K <= 1024) && (S == 1);
+  const bool xreg = kXReg && !kQ8 && !kQ4 && (p.spr == 1) && (p.K <= 1024) && (S == 1);
   float4 xr[8];
   if (xreg) {
     const float4* x4 = reinterpret_cast<const float4*>(xs);
@@ -436,20 +478,22 @@ __device__ inline bool consume_phase(const Ring& r, uint32_t& g, const StagePlan
     const StageDesc s = stage_desc(p, j);
     const int ncols = s.c1 - s.c0, n4 = ncols >> 2;
     const float* st = reinterpret_cast<const float*>(r.buf + (size_t)slot * kStageBytes);
-    if (kQ8) {  // whole 8-bit rows (ncols = Kw words): y = scale * sum q x
+    if (kQ8 || kQ4) {  // whole 8-bit or 4-bit rows (ncols = Kw words): y = scale * sum q x
       const float4* x4 = reinterpret_cast<const float4*>(xs);
       for (int ri = 0; ri < s.nrows; ri += 2) {
         const bool two = ri + 1 < s.nrows;
         const float* r0 = st + (size_t)ri * ncols;
         const float* r1 = r0 + ncols;
+        const int* c0 = reinterpret_cast<const int*>(r0 + 4);
+        const int* c1 = reinterpret_cast<const int*>(r1 + 4);
         float a0, a1 = 0.f;
         if (two) {
-          const float2 t = row2_partial_q8(reinterpret_cast<const int*>(r0 + 4),
-                                           reinterpret_cast<const int*>(r1 + 4), x4, ncols - 4, lane);
+          const float2 t = kQ4 ? row2_partial_q4(c0, c1, x4, ncols - 4, lane)
+                               : row2_partial_q8(c0, c1, x4, ncols - 4, lane);
           a0 = t.x;
           a1 = t.y;
         } else {
-          a0 = row_partial_q8(reinterpret_cast<const int*>(r0 + 4), x4, ncols - 4, lane);
+          a0 = kQ4 ? row_partial_q4(c0, x4, ncols - 4, lane) : row_partial_q8(c0, x4, ncols - 4, lane);
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {

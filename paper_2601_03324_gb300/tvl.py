@@ -78,6 +78,12 @@ def _load():
     L.tvl_quantize_q8.argtypes = [P, P, i32, i32, P]
     L.tvl_gemv_q8.restype = st
     L.tvl_gemv_q8.argtypes = [P, P, P, i32, i32, P]
+    L.tvl_q4_bytes.restype = sz
+    L.tvl_q4_bytes.argtypes = [i32, i32]
+    L.tvl_quantize_q4.restype = st
+    L.tvl_quantize_q4.argtypes = [P, P, i32, i32, P]
+    L.tvl_gemv_q4.restype = st
+    L.tvl_gemv_q4.argtypes = [P, P, P, i32, i32, P]
     L.tvl_gemv_noalloc.restype = st
     L.tvl_gemv_noalloc.argtypes = [P, P, P, i32, i32, P]
     L.tvl_sync.restype = st
@@ -102,6 +108,7 @@ lib = _load()
 EXPORTED = ["tvl_blob_bytes", "tvl_load", "tvl_load_file", "tvl_forward", "tvl_decode_greedy",
             "tvl_forward_batch", "tvl_decode_greedy_batch", "tvl_prefill",
             "tvl_gemv", "tvl_gemv_noalloc", "tvl_q8_bytes", "tvl_quantize_q8", "tvl_gemv_q8",
+            "tvl_q4_bytes", "tvl_quantize_q4", "tvl_gemv_q4",
             "tvl_sync", "tvl_free", "tvl_status_string", "tvl_last_error",
             "tvl_get_info", "tvl_step_times", "tvl_selftest_barrier_timeout"]
 
@@ -170,6 +177,23 @@ def tvl_gemv_q8(Wq8, x, y, d_out: int, d_in: int, stream: int = 0):
     _check(lib.tvl_gemv_q8(ctypes.c_void_p(_addr(Wq8)), ctypes.c_void_p(_addr(x)),
                            ctypes.c_void_p(_addr(y)), int(d_out), int(d_in),
                            ctypes.c_void_p(int(stream))), "tvl_gemv_q8")
+
+
+def tvl_q4_bytes(rows: int, cols: int) -> int:
+    return int(lib.tvl_q4_bytes(int(rows), int(cols)))
+
+
+def tvl_quantize_q4(W, Wq4, rows: int, cols: int, stream: int = 0):
+    """Packed 4-bit rows of W (device addresses)."""
+    _check(lib.tvl_quantize_q4(ctypes.c_void_p(_addr(W)), ctypes.c_void_p(_addr(Wq4)), int(rows),
+                               int(cols), ctypes.c_void_p(int(stream))), "tvl_quantize_q4")
+
+
+def tvl_gemv_q4(Wq4, x, y, d_out: int, d_in: int, stream: int = 0):
+    """y = W' x over packed 4-bit rows (device addresses)."""
+    _check(lib.tvl_gemv_q4(ctypes.c_void_p(_addr(Wq4)), ctypes.c_void_p(_addr(x)),
+                           ctypes.c_void_p(_addr(y)), int(d_out), int(d_in),
+                           ctypes.c_void_p(int(stream))), "tvl_gemv_q4")
 
 
 def tvl_selftest_barrier_timeout(limit_ms: int) -> int:
