@@ -106,3 +106,28 @@ def test_q8_row_bytes_on_the_host(tvl):
     assert tvl.tvl_q8_bytes(32000, 768) == 32000 * 784
     for rows, cols in ((0, 32), (3, 8), (3, 24), (3, 0), (-1, 16)):
         assert tvl.tvl_q8_bytes(rows, cols) == 0
+
+
+def test_q4_row_bytes_and_argument_checks_on_the_host(tvl):
+    assert tvl.tvl_q4_bytes(3, 32) == 3 * 32
+    assert tvl.tvl_q4_bytes(32000, 4096) == 32000 * (16 + 2048)
+    for rows, cols in ((0, 32), (3, 16), (3, 48), (3, 0), (-1, 32)):
+        assert tvl.tvl_q4_bytes(rows, cols) == 0
+    L = tvl.lib
+    # size, null and alignment checks come before any device call
+    assert L.tvl_quantize_q4(None, None, 4, 32, None) == tvl.E_INVAL
+    assert L.tvl_quantize_q4(16, 16, 4, 48, None) == tvl.E_INVAL
+    assert L.tvl_quantize_q4(20, 16, 4, 32, None) == tvl.E_ALIGN
+    assert L.tvl_gemv_q4(None, 16, 16, 4, 32, None) == tvl.E_INVAL
+    assert L.tvl_gemv_q4(16, 16, 16, 4, 40, None) == tvl.E_INVAL
+    assert L.tvl_gemv_q4(16, 24, 16, 4, 32, None) == tvl.E_ALIGN
+    assert L.tvl_gemv_q4(16, 16, 16, 1, 32768, None) == tvl.E_UNSUPPORTED  # row over a stage
+    assert "multiple of 32" in tvl.last_error() or "stage" in tvl.last_error()
+
+
+def test_bench_refuses_q4_decode():
+    import subprocess
+    import sys
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--weights", "q4"],
+                       capture_output=True, text=True, timeout=120)
+    assert r.returncode == 2 and "gemv-sweep" in r.stdout
