@@ -201,7 +201,7 @@ class Model:
     """One decode session of the oracle over a borrowed blob (numpy array kept alive)."""
 
     def __init__(self, cfg: dict, blob: np.ndarray, acc_bits: int = 64, weight_bits: int = 0):
-        """weight_bits 8: every weight matrix as 8-bit codes with row scales."""
+        """weight_bits 8 or 4: every weight matrix as 8-bit or 4-bit codes with row scales."""
         self._blob = blob  # keep alive
         self.cfg = dict(cfg)
         c = make_config(cfg)

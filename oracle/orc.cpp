@@ -218,14 +218,15 @@ struct ModelBase {
   bool tied = false;
 };
 
-// One weight matrix as 8-bit codes and row scales.
+// One weight matrix as codes (qmax levels on each side of zero: 127 for
+// 8-bit rows, 7 for 4-bit ones) and row scales.
 struct QMat {
   std::vector<int8_t> q;
   std::vector<float> s;
-  void make(const float* W, int64_t M, int64_t K) {
+  void make(const float* W, int64_t M, int64_t K, float qmax) {
     q.resize((size_t)(M * K));
     s.resize((size_t)M);
-    quantize_rows(W, M, K, q.data(), s.data());
+    quantize_rows_levels(W, M, K, qmax, q.data(), s.data());
   }
 };
 
@@ -234,7 +235,7 @@ struct Model : ModelBase {
   orc_config c;
   const char* blob;
   Layout L;
-  bool q8 = false;  // weight matrices as 8-bit codes (gains stay float32)
+  bool q8 = false;  // weight matrices as 8-bit or 4-bit codes (gains stay float32)
   std::vector<QMat> qWq, qWk, qWv, qWo, qW1, qW3, qW2;
   QMat qE, qWcls;
   int64_t d, F, V, H, Hkv, hd, kvd, S;
@@ -262,23 +263,23 @@ struct Model : ModelBase {
   }
 
   // Codes of every weight matrix (the embedding table too; it is also the
-  // classifier when tied).
-  void quantize_all() {
+  // classifier when tied), qmax levels on each side of zero.
+  void quantize_all(float qmax) {
     q8 = true;
     const int nl = c.n_layers;
     qWq.resize(nl); qWk.resize(nl); qWv.resize(nl); qWo.resize(nl);
     qW1.resize(nl); qW3.resize(nl); qW2.resize(nl);
     for (int l = 0; l < nl; ++l) {
-      qWq[l].make(T(L.Wq[l]), d, d);
-      qWk[l].make(T(L.Wk[l]), kvd, d);
-      qWv[l].make(T(L.Wv[l]), kvd, d);
-      qWo[l].make(T(L.Wo[l]), d, d);
-      qW1[l].make(T(L.W1[l]), F, d);
-      qW3[l].make(T(L.W3[l]), F, d);
-      qW2[l].make(T(L.W2[l]), d, F);
+      qWq[l].make(T(L.Wq[l]), d, d, qmax);
+      qWk[l].make(T(L.Wk[l]), kvd, d, qmax);
+      qWv[l].make(T(L.Wv[l]), kvd, d, qmax);
+      qWo[l].make(T(L.Wo[l]), d, d, qmax);
+      qW1[l].make(T(L.W1[l]), F, d, qmax);
+      qW3[l].make(T(L.W3[l]), F, d, qmax);
+      qW2[l].make(T(L.W2[l]), d, F, qmax);
     }
-    qE.make(T(L.E), V, d);
-    if (!tied) qWcls.make(T(L.Wcls), V, d);
+    qE.make(T(L.E), V, d, qmax);
+    if (!tied) qWcls.make(T(L.Wcls), V, d, qmax);
   }
   void mv(const std::vector<QMat>& qm, const std::vector<int64_t>& off, int l, const Acc* xin,
           Acc* yout, int64_t M, int64_t K) {
@@ -384,7 +385,7 @@ void* orc_model_new_fmt(const orc_config* cfg, const void* blob, size_t blob_byt
   if (!err) err = &dummy;
   *err = 0;
   if (!config_ok(cfg) || !blob || (acc_bits != 32 && acc_bits != 64) ||
-      (weight_bits != 0 && weight_bits != 8)) {
+      (weight_bits != 0 && weight_bits != 8 && weight_bits != 4)) {
     *err = 1;
     return nullptr;
   }
@@ -414,9 +415,10 @@ void* orc_model_new_fmt(const orc_config* cfg, const void* blob, size_t blob_byt
   }
   if (!m) { *err = 4; return nullptr; }
   m->tied = tied;
-  if (weight_bits == 8) {
-    if (acc_bits == 64) static_cast<Model<double>*>(m)->quantize_all();
-    else static_cast<Model<float>*>(m)->quantize_all();
+  if (weight_bits != 0) {
+    const float qmax = weight_bits == 8 ? 127.0f : 7.0f;
+    if (acc_bits == 64) static_cast<Model<double>*>(m)->quantize_all(qmax);
+    else static_cast<Model<float>*>(m)->quantize_all(qmax);
   }
   return m;
 }

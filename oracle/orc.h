@@ -42,9 +42,9 @@ int64_t orc_tensor_offset(const orc_config* cfg, int tied, int which, int layer)
  * Returns NULL and sets *err (1 invalid config, 2 size mismatch, 4 no memory). */
 void* orc_model_new(const orc_config* cfg, const void* blob, size_t blob_bytes,
                     int acc_bits, int* err);
-/* Same, with every weight matrix replaced by 8-bit codes and row scales
- * (weight_bits 8; 0 keeps float32), quantized at construction as
- * orc_quantize_rows_q8 defines. */
+/* Same, with every weight matrix replaced by codes and row scales, quantized
+ * at construction as orc_quantize_rows_q8 (weight_bits 8) or
+ * orc_quantize_rows_q4 (weight_bits 4) defines; 0 keeps float32. */
 void* orc_model_new_fmt(const orc_config* cfg, const void* blob, size_t blob_bytes,
                         int acc_bits, int weight_bits, int* err);
 /* One decode step (token at position pos); writes vocab_size logits.

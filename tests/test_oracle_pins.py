@@ -419,9 +419,9 @@ def test_q4_code_is_the_nearest_of_the_15_levels_by_brute_force():
             assert d[int(q[i, j]) + 7] <= d.min() * (1 + 1e-6) + 1e-15
 
 
-def _representable_blob(cfg, seed):
-    """A blob whose every weight matrix row is k * 2^-12 with integer |k| <= 127
-    and some |k| == 127: its 8-bit codes and scales are exact."""
+def _representable_blob(cfg, seed, kmax=127):
+    """A blob whose every weight matrix row is k * 2^-12 with integer |k| <= kmax
+    and some |k| == kmax: its codes with kmax levels and its scales are exact."""
     blob = synth.make_blob(cfg, seed=seed)
     names = ["Wq", "Wk", "Wv", "Wo", "W1", "W3", "W2"]
     mats = [("E", -1)] + [(n, l) for l in range(cfg["n_layers"]) for n in names]
@@ -429,8 +429,8 @@ def _representable_blob(cfg, seed):
         mats.append(("Wcls", -1))
     for (n, l) in mats:
         T = synth.tensor(blob, cfg, n, l)
-        k = np.clip(np.rint(T * 4096.0), -127, 127)
-        k[:, 0] = np.where(k[:, 0] < 0, -127, 127)
+        k = np.clip(np.rint(T * 4096.0 * kmax / 127), -kmax, kmax)
+        k[:, 0] = np.where(k[:, 0] < 0, -kmax, kmax)
         T[...] = (k / 4096.0).astype(np.float32)
     return blob
 
@@ -453,3 +453,27 @@ def test_q8_model_differs_from_float_model_by_quantization_only():
     lq = oracle.Model(cfg, blob, weight_bits=8).forward(1, 0)
     rel = np.abs(lq - lf).max() / np.abs(lf).max()
     assert 1e-5 < rel < 5e-2  # the codes change the result, by about the code step
+
+
+@pytest.mark.parametrize("tied", [1, 0])
+def test_q4_model_equals_float_model_on_exactly_representable_weights(tied):
+    cfg = dict(synth.model_config("tiny"), n_layers=2, vocab_size=500, max_seq=8,
+               shared_classifier=tied)
+    blob = _representable_blob(cfg, 7, kmax=7)
+    mf = oracle.Model(cfg, blob)
+    mq = oracle.Model(cfg, blob, weight_bits=4)
+    for pos, tok in enumerate([3, 17, 499, 0, 250]):
+        assert np.array_equal(mq.forward(tok, pos), mf.forward(tok, pos))
+
+
+def test_q4_model_is_coarser_than_q8_and_differs_by_quantization_only():
+    cfg = dict(synth.model_config("tiny"), n_layers=2, vocab_size=500, max_seq=8)
+    blob = synth.make_blob(cfg, seed=6)
+    lf = oracle.Model(cfg, blob).forward(1, 0)
+    l8 = oracle.Model(cfg, blob, weight_bits=8).forward(1, 0)
+    l4 = oracle.Model(cfg, blob, weight_bits=4).forward(1, 0)
+    r8 = np.abs(l8 - lf).max() / np.abs(lf).max()
+    r4 = np.abs(l4 - lf).max() / np.abs(lf).max()
+    assert 4 * r8 < r4 < 1.0  # 15 levels instead of 255: a far larger code step
+    with pytest.raises(ValueError):
+        oracle.Model(cfg, blob, weight_bits=5)
