@@ -57,6 +57,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--gemv-sweep", action="store_true", help="GEMV GB/s per shape instead")
+    ap.add_argument("--hot", action="store_true",
+                    help="with --gemv-sweep: one copy of W, so that W stays in L2 when it fits")
     ap.add_argument("--batch", type=int, default=1, choices=[1, 2, 3, 4],
                     help="sequences decoded together per launch (tvl_decode_greedy_batch)")
     return ap.parse_args()
@@ -305,7 +307,7 @@ def gemv_sweep(args):
                   "q4": (tvl.tvl_q4_bytes, tvl.tvl_quantize_q4, tvl.tvl_gemv_q4)}.get(args.weights)
         wbytes = packed[0](M, K) if packed else 4 * M * K
         nbytes = wbytes + 4 * (M + K)
-        copies = max(1, math.ceil(3 * l2 / wbytes))
+        copies = 1 if args.hot else max(1, math.ceil(3 * l2 / wbytes))
         if packed:  # packed 8-bit or 4-bit rows of W, one copy per rotation slot
             dW1 = torch.from_numpy(W).cuda()
             dW = torch.empty((copies, wbytes), dtype=torch.uint8, device="cuda")
@@ -336,13 +338,17 @@ def gemv_sweep(args):
             e1.record(s)
         e1.synchronize()
         us = e0.elapsed_time(e1) * 1000.0 / reps
-        out.append({"shape": [M, K], "us": us, "GB/s": nbytes / us / 1e3, "cold_copies": copies})
+        out.append({"shape": [M, K], "us": us, "GB/s": nbytes / us / 1e3,
+                    "copies": copies, "fits_l2": wbytes <= l2})
         del dW, g
     peak, src = measured_peaks()
     for o in out:
         o["frac_of_" + src + "_hbm"] = o["GB/s"] / peak
-    print(json.dumps({"gemv_sweep": out, "weights": args.weights, "peak_gbs": peak,
-                      "peak_source": src}), flush=True)
+    mode = ("hot: one copy of W, resident in L2 when it fits (its GB/s is then an L2 figure, "
+            "not an HBM one)" if args.hot else
+            "cold: W rotated over copies totalling 3x L2, so every call reads it from HBM")
+    print(json.dumps({"gemv_sweep": out, "weights": args.weights, "mode": mode,
+                      "peak_gbs": peak, "peak_source": src}), flush=True)
 
 
 def main():
