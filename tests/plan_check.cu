@@ -4,13 +4,16 @@
 // exactly once, every copy stays inside its matrix, holds at most one stage,
 // starts on a 16-byte boundary and has a size that is a multiple of 16 bytes
 // (the bulk-copy rules), row pairs stay whole within one CTA, and deferred
-// partials fit the shared scratch. Prints "ok <plans>" or FAIL lines.
+// partials fit the shared scratch. Also the attention split (att_split): the
+// chunks of every position cover positions 0..pos exactly, none is empty or
+// longer than the score scratch, and with B sequences no head gets more
+// chunks than the record buffer holds. Prints "ok <plans>" or FAIL lines.
 #include <algorithm>
 #include <cstdio>
 #include <utility>
 #include <vector>
 
-#include "../paper_2601_03324_gb300/csrc/stream_gemv.cuh"
+#include "../paper_2601_03324_gb300/csrc/decode_kernel.cuh"
 
 using namespace tvl;
 
@@ -90,6 +93,39 @@ static int split_for(int M, int K, int G) {
   return S;
 }
 
+// The record buffer holds, per (sequence, head), the most chunks one sequence's
+// head gets at any position (the arena's rule).
+static int nch_cap_for(int S, int H, int G) {
+  int cap = 1;
+  for (int pos = 0; pos < S; ++pos) {
+    int nch, clen;
+    att_split(pos, H, G, &nch, &clen);
+    cap = std::max(cap, nch);
+  }
+  return cap;
+}
+
+static void check_attention(int S, int H, int G) {
+  const int cap = nch_cap_for(S, H, G);
+  for (int B = 1; B <= 4; ++B)
+    for (int pos = 0; pos < S; ++pos) {
+      int nch, clen;
+      att_split(pos, H * B, G, &nch, &clen);
+      CHECK(nch >= 1 && nch <= cap, "S=%d H=%d G=%d B=%d pos=%d: %d chunks, capacity %d", S, H, G,
+            B, pos, nch, cap);
+      CHECK(clen >= 1 && clen <= kAttMaxChunk, "pos=%d: chunk of %d positions", pos, clen);
+      int covered = 0;
+      for (int c = 0; c < nch; ++c) {
+        const int t0 = c * clen, t1 = std::min(t0 + clen, pos + 1);
+        CHECK(t0 == covered && t1 > t0, "S=%d H=%d G=%d B=%d pos=%d chunk %d: [%d, %d)", S, H, G,
+              B, pos, c, t0, t1);
+        covered = t1;
+      }
+      CHECK(covered == pos + 1, "pos=%d: chunks end at %d", pos, covered);
+      ++nplans;
+    }
+}
+
 int main() {
   const Shape shapes[] = {{"tiny", 288, 768, 6, 6, 32000},     {"110m", 768, 2048, 12, 12, 32000},
                           {"7b", 4096, 11008, 32, 32, 32000},  {"small", 64, 96, 4, 4, 1000},
@@ -137,6 +173,9 @@ int main() {
       if (p0.spr > 1 && ((nv + G - 1) / G) * p0.spr > kMaxSegParts) continue;  // per-row kernel
       check(what, nv, mk[1] / S, G, 1, 1);
     }
+  const int att[][2] = {{256, 6}, {1024, 12}, {2048, 32}, {64, 4}, {64, 1}, {4096, 2}};
+  for (auto& sh : att)
+    for (int G : Gs) check_attention(sh[0], sh[1], G);
   if (fails) {
     printf("%d failures\n", fails);
     return 1;
