@@ -27,6 +27,7 @@ import math
 import os
 import statistics
 import subprocess
+import tempfile
 import sys
 import time
 
@@ -142,19 +143,26 @@ class Clocks:
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
     def __init__(self, dev_index: int, uuid: str | None):
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
-        os.makedirs(os.path.dirname(self.path), exist_ok=True)
+        fd, self.path = tempfile.mkstemp(prefix="tvl_clocks_", suffix=".csv")
+        self.f = os.fdopen(fd, "w")
         cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
                "-lms", "50"]
         cmd += ["-i", uuid] if uuid else ["-i", str(dev_index)]
         try:
-            self.f = open(self.path, "w")
             self.p = subprocess.Popen(cmd, stdout=self.f, stderr=subprocess.DEVNULL)
         except OSError:
             self.p = None
 
+    def _discard(self):
+        self.f.close()
+        try:
+            os.remove(self.path)
+        except OSError:
+            pass
+
     def stop(self, t0: float, t1: float):
         if self.p is None:
+            self._discard()
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
         time.sleep(0.12)
         self.p.terminate()
@@ -163,8 +171,11 @@ class Clocks:
         except subprocess.TimeoutExpired:
             self.p.kill()
         self.f.close()
+        with open(self.path) as fh:
+            lines = fh.readlines()
+        self._discard()
         rows = []
-        for line in open(self.path):
+        for line in lines:
             parts = [x.strip() for x in line.split(",")]
             if len(parts) < 9:
                 continue
