@@ -248,6 +248,102 @@ def test_kv_cache_attention_averages_all_positions_up_to_current():
     assert np.array_equal(m.forward(1, 1), lg1)
 
 
+def _unit_kappa(c: float, d: int, eps: float = 1e-5) -> float:
+    """RMSNorm output of a one-hot row c * e_t with unit gain: kappa * e_t."""
+    return c * (1.0 / math.sqrt(c * c / d + eps))
+
+
+def test_rope_turns_q_and_k_at_their_own_positions_and_leaves_v_alone():
+    # §2.1: RoPE rotates q and k (not v), and the cached key of position 0 keeps
+    # the rotation of position 0. One head of width 4; pair (0, 1) turns by p
+    # radians at position p. Token 2 at position 0, token 3 at position 1, each
+    # embedding a one-hot row, so x_b = kappa * e_t:
+    #   q(pos 1) = kappa*qa*e0, turned by 1 -> kappa*qa*(cos 1, sin 1)
+    #   k(pos 0) = kappa*kb*e0 (angle 0),  k(pos 1) = kappa*kb*e1 turned by 1
+    #   v(pos 0) = kappa*gv*e0,            v(pos 1) = kappa*gv*e1 (never turned)
+    # Scores: s0 = kappa^2 qa kb cos(1) / 2 and s1 = 0 (q and k(pos 1) turn by
+    # the same angle and start orthogonal). With Wo = I, zero FFN and Wcls = I,
+    # the logits are proportional to x = (kappa gv w0, kappa gv w1, 0, c).
+    # A key cached before its rotation, a key turned at the reader's position,
+    # no rotation at all, or a rotated v each change lg0 / lg1 = w0 / w1.
+    c, qa, kb, gv = 10.0, 0.5, 1.0, 1.0
+    cfg = _tiny_cfg()
+    E = np.zeros((4, 4), np.float32)
+    E[2, 2] = c
+    E[3, 3] = c
+    Wq = np.zeros((4, 4), np.float32)
+    Wq[0, 3] = qa
+    Wk = np.zeros((4, 4), np.float32)
+    Wk[0, 2] = kb
+    Wk[1, 3] = kb
+    Wv = np.zeros((4, 4), np.float32)
+    Wv[0, 2] = gv
+    Wv[1, 3] = gv
+    blob = _blob(cfg, E=E, Wq0=Wq, Wk0=Wk, Wv0=Wv, Wo0=np.eye(4), Wcls=np.eye(4))
+    m = oracle.Model(cfg, blob)
+    kap = _unit_kappa(c, 4)
+    lg0 = m.forward(2, 0)  # one position: the output is v(pos 0) itself
+    assert abs(lg0[0] / lg0[2] - kap * gv / c) < 1e-12 and lg0[1] == 0.0 and lg0[3] == 0.0
+    lg = m.forward(3, 1)
+    s0 = (kap * qa) * (kap * kb) * math.cos(1.0) / 2.0
+    w0 = 1.0 / (1.0 + math.exp(-s0))
+    w1 = 1.0 - w0
+    assert abs(lg[0] / lg[1] - w0 / w1) < 1e-12 * (w0 / w1)
+    assert abs(lg[0] / lg[3] - kap * gv * w0 / c) < 1e-12
+    assert lg[2] == 0.0
+
+
+def test_each_head_reads_its_own_q_k_v_slices_and_writes_its_own_output():
+    # Two heads of width 2 (H = Hkv = 2): head h reads q, k, v elements
+    # [2h, 2h + 2) and writes o elements [2h, 2h + 2). Token 0 at position 0,
+    # token 1 at position 1, one-hot embeddings (x_b = kappa * e_t).
+    #   head 0: q = kappa*Qw*(1, 0), head 1: q = -0.75*kappa*Qw*(1, 0) (pos 1)
+    #   both heads: k(pos 0) = kappa*kw*(1, 0), k(pos 1) = kappa*Kw*(1, 0)
+    #   v(pos 0) = kappa*gw*e3 (head 1's slice), v(pos 1) = kappa*gw*e0 (head 0's)
+    # Head 0 leans to position 1, head 1 to position 0 (its q points the other
+    # way), so o = (kappa gw w1[0], 0, 0, kappa gw w0[1]) with w the softmax
+    # weights of each head; q, k turn by the same angle at position 1 and k of
+    # position 0 not at all, so s0 = a * kw * cos(1) / sqrt(2), s1 = a * Kw / sqrt(2)
+    # with a = the head's q length times kappa. Heads reading head 0's q, one
+    # kv head for all, or outputs written to the wrong slice break lg3/lg1 or lg2.
+    c, Qw, kw, Kw, gw = 10.0, 1.0, 0.5, 1.0, 1.0
+    cfg = _tiny_cfg(n_heads=2, n_kv_heads=2)
+    E = np.zeros((4, 4), np.float32)
+    E[0, 0] = c
+    E[1, 1] = c
+    Wq = np.zeros((4, 4), np.float32)
+    Wq[0, 1] = Qw
+    Wq[2, 1] = -0.75 * Qw
+    Wk = np.zeros((4, 4), np.float32)
+    Wk[0, 0] = kw
+    Wk[2, 0] = kw
+    Wk[0, 1] = Kw
+    Wk[2, 1] = Kw
+    Wv = np.zeros((4, 4), np.float32)
+    Wv[3, 0] = gw
+    Wv[0, 1] = gw
+    blob = _blob(cfg, E=E, Wq0=Wq, Wk0=Wk, Wv0=Wv, Wo0=np.eye(4), Wcls=np.eye(4))
+    m = oracle.Model(cfg, blob)
+    kap = _unit_kappa(c, 4)
+    lg0 = m.forward(0, 0)  # one position: head 1's output is its slice of v(pos 0)
+    assert abs(lg0[3] / lg0[0] - kap * gw / c) < 1e-12 and lg0[1] == 0.0 and lg0[2] == 0.0
+    lg = m.forward(1, 1)
+
+    def weights(qlen):
+        a = kap * qlen * kap
+        s0 = a * kw * math.cos(1.0) / math.sqrt(2.0)
+        s1 = a * Kw / math.sqrt(2.0)
+        w1 = 1.0 / (1.0 + math.exp(s0 - s1))
+        return 1.0 - w1, w1
+
+    _, w1_h0 = weights(Qw)
+    w0_h1, _ = weights(-0.75 * Qw)
+    assert w1_h0 > 0.8 and w0_h1 > 0.7  # the heads lean to different positions
+    assert abs(lg[0] / lg[1] - kap * gw * w1_h0 / c) < 1e-12
+    assert abs(lg[3] / lg[1] - kap * gw * w0_h1 / c) < 1e-12
+    assert lg[2] == 0.0
+
+
 def test_zero_output_projections_make_the_layer_an_identity():
     cfg1 = dict(synth.model_config("tiny"), n_layers=1, vocab_size=512)
     blob1 = synth.make_blob(cfg1, seed=7)
