@@ -2,18 +2,26 @@
 """Benchmark: batch-1 FP32 decode tokens/s of the 110M Llama-2-shape model.
 
 A step is one decode step (all layers + classifier + greedy argmax) for one
-token. The timed region runs K steps as greedy sequences of 256 steps from
-token 1 (the paper's 256-token run), each sequence one launch of the
-persistent decode kernel, with the weights resident in HBM. Weights streamed
-per step (438 MB) exceed L2 (~126 MB), so no L2 flush is needed between steps.
+token. The workload is greedy 256-step sequences from token 1 (the paper's
+256-token run) with the weights resident in HBM. K timed steps are whole
+sequences (one launch of the persistent decode kernel each) and, for the
+K mod 256 steps left, one window of consecutive positions centred on the
+sequence, so the timed steps have the sequence's mean KV length; an untimed
+launch first decodes the whole sequence, which fills the KV cache and gives
+the token each window starts from (greedy decoding is deterministic). The
+positions timed are in config.positions; full_sequence times one whole
+sequence on its own. Weights streamed per step (438 MB) exceed L2, so no L2
+flush is needed between steps.
 
 Printed JSON line (rank 0): value = tokens/s over all ranks; e2e = the same
 metric through tvl_forward with host logits (token in, 128 KB of logits out,
-host argmax, every step); roofline of the decode kernel against the measured
-HBM copy bandwidth; cpu_baseline = the CPU oracle on the host cores.
+host argmax, every step, the same positions); roofline of the decode kernel
+against the measured HBM copy bandwidth; cpu_baseline = the CPU oracle with
+float accumulators (the paper's scalar baseline) on one host core;
+cpu_baseline_paper_method = the paper's NEON GEMV and RMSNorm on one host core.
 
 --impl reference times the CPU oracle (the only reference this paper has; it
-publishes no code) on the same workload.
+publishes no code) on the same workload and positions.
 
 Multi-GPU (torchrun): replicas only — each rank decodes its own sequences; no
 collective on the data path. value = all ranks' tokens / max rank time.
@@ -199,11 +207,42 @@ class Clocks:
                 "power_w": statistics.median(pws) if pws else None}
 
 
-def cpu_oracle_rate(cfg, blob, seconds: float, weight_bits: int = 0):
-    """The CPU oracle (double accumulators, one thread) decoding greedily from
-    token 1 for about `seconds`; tokens/s."""
-    import oracle
-    m = oracle.Model(cfg, blob, 64, weight_bits=weight_bits)
+def timed_windows(seq: int, k: int, pos0: int):
+    """(first position, steps) of each launch that times k steps of the
+    workload's seq-step sequences from pos0: whole sequences, then the steps
+    left as one window centred on the sequence, so that the timed steps have
+    the sequence's mean KV length."""
+    wins = [(pos0, seq)] * (k // seq)
+    r = k % seq
+    if r:
+        wins.append((pos0 + (seq - r) // 2, r))
+    return wins
+
+
+def window_starts(wins, pos0: int, first, fill):
+    """Start token(s) of each window: the sequence's first token(s) at pos0,
+    else the greedy token(s) at that position from the fill run (fill[s] is
+    the argmax after step s of the sequence)."""
+    out = []
+    for (p, n) in wins:
+        out.append(list(first) if p == pos0 else [int(t) for t in np.atleast_1d(fill[p - pos0 - 1])])
+    return out
+
+
+def positions_of(wins):
+    """config.positions: the distinct [first, last] position ranges timed."""
+    seen = []
+    for (p, n) in wins:
+        r = [p, p + n - 1]
+        if r not in seen:
+            seen.append(r)
+    return seen
+
+
+def cpu_decode_rate(make, cfg, seconds: float):
+    """A CPU decoder (make() -> object with forward(token, pos)) decoding
+    greedily from token 1 for about `seconds`; tokens/s, steps, seconds."""
+    m = make()
     t, n = 1, 0
     t0 = time.perf_counter()
     while True:
@@ -216,31 +255,94 @@ def cpu_oracle_rate(cfg, blob, seconds: float, weight_bits: int = 0):
     return n / el, n, el
 
 
+def streamed_bytes_of(cfg: dict, weight_bits: int = 0) -> int:
+    """Weight bytes one decode step reads: every matrix and gain of every
+    layer, one embedding row, the final gain and the classifier (8-bit rows:
+    16 + K bytes per row)."""
+    d, F, L, V = cfg["dim"], cfg["hidden_dim"], cfg["n_layers"], cfg["vocab_size"]
+    kvd = cfg["n_kv_heads"] * (d // cfg["n_heads"])
+    if weight_bits == 8:
+        return (L * ((d + 2 * kvd) * (16 + d) + d * (16 + d) + 2 * F * (16 + d) + d * (16 + F)
+                     + 8 * d) + V * (16 + d) + (16 + d) + 4 * d)
+    return 4 * (L * ((d + 2 * kvd) * d + d * d + 3 * F * d + 2 * d) + V * d + 2 * d)
+
+
+def l2_statement(streamed: int) -> str:
+    """How the timed steps relate to L2 (the timing rule: inputs larger than L2,
+    or say that they are not). GB300's L2 holds about 126 MB."""
+    if streamed > 140e6:
+        return (f"inputs larger than L2: every step streams {streamed / 1e6:.1f} MB of weights "
+                f"(GB300 L2: about 126 MB), so no flush is needed between steps")
+    return (f"weights fit in L2 ({streamed / 1e6:.1f} MB streamed per step; GB300 L2: about "
+            f"126 MB) and are not flushed between the steps of a launch: the roofline against "
+            f"HBM bandwidth understates this workload's bound (see roofline.l2)")
+
+
+def workload_config(name, cfg, batch=1, weights="f32", positions=None):
+    """The config object of the JSON line; both arms build it from the same
+    arguments, so that the driver's same-config check holds."""
+    desc = {"110m": "110M Llama-2-shape FP32 decoder (d768 L12 H12 F2048 V32000, tied), "
+                    "batch 1, greedy 256-step sequences from token 1",
+            "110m-long": "110M Llama-2-shape FP32 decoder (d768 L12 H12 F2048 V32000, tied), "
+                         "batch 1, KV cache filled by one prefill of 896 prompt tokens "
+                         "(uniform in [3, 31999], seed 3), greedy 128-step sequences at "
+                         "positions 896..1023",
+            "tiny": "tiny Llama-2-shape FP32 decoder (d288 L6 H6 F768 V32000, untied), batch 1, "
+                    "greedy 64-step sequences from token 1",
+            "7b": "7B Llama-2-shape FP32 decoder (d4096 L32 H32 F11008 V32000, untied), batch 1, "
+                  "greedy 16-step sequences from token 1"}[name]
+    seq = 128 if name == "110m-long" else min(cfg["steps"], cfg["max_seq"])
+    if batch > 1:
+        desc = desc.replace("batch 1, greedy", f"{batch} sequences per launch (first tokens "
+                            f"{BATCH_STARTS[:batch]}), greedy").replace(" from token 1", "")
+    return {"workload": desc, "seq_steps": seq, "batch": batch,
+            "weights_seed": cfg["seed"], "parallelism": "replicas", "weights": weights,
+            "positions": positions,
+            "l2": l2_statement(streamed_bytes_of(cfg, 8 if weights == "q8" else 0))}
+
+
 def run_reference(args, cfg, rank, world):
+    """The CPU oracle (double accumulators, one host core) on the same
+    positions as the GPU arm: an untimed greedy fill up to the last window's
+    start, the warm-up steps, then the timed windows (or, when whole steps
+    would take longer than about 150 s, the same fraction of every weight
+    matrix's rows per step, scaled to whole steps)."""
     if rank != 0:
         return 0
     from paper_2601_03324_gb300 import synth
     import oracle
     blob = synth.make_blob(cfg)
     m = oracle.Model(cfg, blob, 64)
-    t = 1
+    seq, pos0 = min(cfg["steps"], cfg["max_seq"]), 0
+    tok0 = 1
+    if args.workload == "110m-long":
+        prompt = synth.long_context_tokens()
+        for p, t in enumerate(prompt):
+            lg = m.forward(int(t), p)
+        tok0, pos0, seq = int(np.argmax(lg)), len(prompt), cfg["max_seq"] - len(prompt)
+    wins = timed_windows(seq, args.steps, pos0)
+    fill, t = [], tok0
+    for p in range(pos0, max(p for p, _ in wins)):
+        t = int(np.argmax(m.forward(t, p)))
+        fill.append(t)
+    starts = window_starts(wins, pos0, [tok0], fill)
+    wp, wn = wins[-1]
     for s in range(args.warmup):
-        t = int(np.argmax(m.forward(t, s % cfg["max_seq"])))
-    # size each step so the whole run stays within ~150 s: a whole token when
-    # that fits, else the same fraction of every weight matrix's rows
+        if s % wn == 0:
+            t = starts[-1][0]
+        t = int(np.argmax(m.forward(t, wp + s % wn)))
     t0 = time.perf_counter()
-    m.forward(t, 0)
+    m.forward(starts[0][0], wins[0][0])
     t_tok = time.perf_counter() - t0
     frac = min(1.0, 150.0 / max(1e-9, args.steps * t_tok))
     t0 = time.perf_counter()
     if frac >= 1.0:
-        pos = 0
-        for s in range(args.steps):
-            t = int(np.argmax(m.forward(t, pos)))
-            pos = (pos + 1) % SEQ
-            if pos == 0:
-                t = 1
-        sample = f"{args.steps} whole decode steps of the workload (greedy, 256-step sequences)"
+        for (p, n), st in zip(wins, starts):
+            t = st[0]
+            for i in range(n):
+                t = int(np.argmax(m.forward(t, p + i)))
+        sample = (f"{args.steps} whole decode steps at the GPU arm's positions "
+                  f"{positions_of(wins)} (greedy, after an untimed fill)")
     else:
         from paper_2601_03324_gb300 import synth as sy
         mats = [(n, l) for l in range(cfg["n_layers"])
@@ -260,49 +362,16 @@ def run_reference(args, cfg, rank, world):
     line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "tokens/s",
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1000.0 * el / (args.steps * frac), "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": val / PAPER_TOKS, "dtype": "f64",
-            "data": "synthetic",
-            "config": dict(workload_config(args.workload, cfg),
-                           l2="the oracle runs on the host cores: no GPU cache is involved"),
+            "scaling": "weak",
+            "vs_baseline": val / PAPER_TOKS if args.workload == "110m" else None, "dtype": "f64",
+            "data": "synthetic (seeded N(0, 0.02) weights)",
+            "config": workload_config(args.workload, cfg, 1, args.weights, positions_of(wins)),
             "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0
-
-
-def l2_statement(streamed_bytes=None, l2_bytes=None) -> str:
-    """How the timed steps relate to L2 (the timing rule: inputs larger than L2,
-    or say that they are not)."""
-    if streamed_bytes is None or not l2_bytes:
-        return "inputs larger than L2: every step streams all weights (> L2 size)"
-    if streamed_bytes > l2_bytes:
-        return (f"inputs larger than L2: every step streams {streamed_bytes / 1e6:.1f} MB of "
-                f"weights, L2 {l2_bytes / 1e6:.1f} MB")
-    return (f"weights fit in L2 ({streamed_bytes / 1e6:.1f} MB streamed per step, L2 "
-            f"{l2_bytes / 1e6:.1f} MB) and are not flushed between the steps of a launch: "
-            f"the roofline against HBM bandwidth understates this workload's bound")
-
-
-def workload_config(name, cfg, batch=1, streamed_bytes=None, l2_bytes=None):
-    desc = {"110m": "110M Llama-2-shape FP32 decoder (d768 L12 H12 F2048 V32000, tied), "
-                    "batch 1, greedy 256-step sequences from token 1",
-            "110m-long": "110M Llama-2-shape FP32 decoder (d768 L12 H12 F2048 V32000, tied), "
-                         "batch 1, KV cache filled by one prefill of 896 prompt tokens "
-                         "(uniform in [3, 31999], seed 3), greedy 128-step sequences at "
-                         "positions 896..1023",
-            "tiny": "tiny Llama-2-shape FP32 decoder (d288 L6 H6 F768 V32000, untied), batch 1, "
-                    "greedy 64-step sequences from token 1",
-            "7b": "7B Llama-2-shape FP32 decoder (d4096 L32 H32 F11008 V32000, untied), batch 1, "
-                  "greedy 16-step sequences from token 1"}[name]
-    seq = 128 if name == "110m-long" else min(cfg["steps"], cfg["max_seq"])
-    if batch > 1:
-        desc = desc.replace("batch 1, greedy", f"{batch} sequences per launch (first tokens "
-                            f"{BATCH_STARTS[:batch]}), greedy").replace(" from token 1", "")
-    return {"workload": desc, "seq_steps": seq, "batch": batch,
-            "weights_seed": cfg["seed"], "parallelism": "replicas",
-            "l2": l2_statement(streamed_bytes, l2_bytes)}
 
 
 def gemv_sweep(args):
@@ -418,28 +487,34 @@ def main():
         tok0, pos0 = int(np.argmax(host)), len(prompt)
         seq = cfg["max_seq"] - pos0
 
-    def run_steps(k, events=None):
-        """k decode steps as greedy sequences of `seq` steps (one launch each)."""
-        launches = 0
-        done = 0
-        while done < k:
-            n = min(seq, k - done)
+    first = [tok0] if B == 1 else BATCH_STARTS[:B]
+
+    def launch(starts, p, n):
+        if B == 1:
+            return model.decode_greedy(starts[0], p, n, tokens=False)
+        return model.decode_greedy_batch(starts, p, n, tokens=False)
+
+    def run_windows(wins, starts, events=None):
+        """One launch per window; CUDA events around each when asked."""
+        for (p, n), st in zip(wins, starts):
             if events is not None:
                 e0 = torch.cuda.Event(enable_timing=True)
                 e0.record(stream)
-            if B == 1:
-                model.decode_greedy(tok0, pos0, n, tokens=False)
-            else:
-                model.decode_greedy_batch(BATCH_STARTS[:B], pos0, n, tokens=False)
+            launch(st, p, n)
             if events is not None:
                 e1 = torch.cuda.Event(enable_timing=True)
                 e1.record(stream)
-                events.append((e0, e1, n))
-            done += n
-            launches += 1
-        return launches
+                events.append((e0, e1, p, n))
+        return len(wins)
 
-    run_steps(max(3, args.warmup))
+    # untimed: the whole sequence once (fills the KV cache, gives the greedy
+    # tokens the windows start from), then the warm-up steps
+    fill = (model.decode_greedy(tok0, pos0, seq) if B == 1 else
+            model.decode_greedy_batch(first, pos0, seq))
+    wins = timed_windows(seq, args.steps, pos0)
+    starts = window_starts(wins, pos0, first, fill)
+    wwins = timed_windows(seq, max(3, args.warmup), pos0)
+    run_windows(wwins, window_starts(wwins, pos0, first, fill))
     model.sync()
     props = torch.cuda.get_device_properties(local_rank)
     uuid = getattr(props, "uuid", None)
@@ -454,7 +529,7 @@ def main():
     start = torch.cuda.Event(enable_timing=True)
     end = torch.cuda.Event(enable_timing=True)
     start.record(stream)
-    launches = run_steps(args.steps, ev)
+    launches = run_windows(wins, starts, ev)
     end.record(stream)
     model.sync()
     torch.cuda.synchronize()
@@ -465,26 +540,66 @@ def main():
     clk = clocks.stop(t_wall0, t_wall1)
     el_ms = max_over_ranks(el_ms, world, "cuda")
 
-    # per-launch roofline of the decode kernel (full-length launches)
-    full = [(a.elapsed_time(b), n) for (a, b, n) in ev]
-    launch_ms = statistics.mean(t for t, n in full)
-    n_typ = full[0][1]
-    bytes_launch = sum(step_bytes(cfg, info.streamed_bytes, pos0 + p, B) for p in range(n_typ))
+    # roofline of the decode kernel: algorithmic bytes of every timed launch
+    # over the sum of their CUDA-event durations
+    per = [(a.elapsed_time(b), p, n) for (a, b, p, n) in ev]
+    kern_ms = sum(t for t, p, n in per)
+    bytes_timed = sum(step_bytes(cfg, info.streamed_bytes, p + i, B)
+                      for (t, p, n) in per for i in range(n))
+    bytes_launch = bytes_timed / len(per)
     peak, peak_src = measured_peaks()
-    achieved = bytes_launch / (statistics.mean(t for t, n in full if n == n_typ) * 1e-3) / 1e9
+    achieved = bytes_timed / (kern_ms * 1e-3) / 1e9
     traffic = committed_traffic(args.workload + ("_q8" if args.weights == "q8" else "") +
                                 (f"_b{B}" if B > 1 else ""), bytes_launch)
-    steps_ns = model.step_times(n_typ).astype(np.float64)
-    dts = np.diff(steps_ns) / 1e3 if n_typ > 1 else np.array([launch_ms * 1e3])
 
-    # end to end through the public API: token(s) in, host logits out, host argmax
+    # one whole sequence on its own (not part of the timed region)
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    f0.record(stream)
+    launch(first, pos0, seq)
+    f1.record(stream)
+    model.sync()
+    full_ms = f0.elapsed_time(f1)
+    full_seq = {"positions": [pos0, pos0 + seq - 1], "ms_per_step": full_ms / seq,
+                "tokens_per_s": B * seq / (full_ms * 1e-3),
+                "roofline_frac": sum(step_bytes(cfg, info.streamed_bytes, pos0 + i, B)
+                                     for i in range(seq)) / (full_ms * 1e-3) / 1e9 / peak,
+                "note": "one launch of the whole greedy sequence after the timed region "
+                        "(CUDA events on the model's stream)"}
+    steps_ns = model.step_times(seq).astype(np.float64)
+    dts = np.diff(steps_ns) / 1e3 if seq > 1 else np.array([full_ms * 1e3])
+
+    # L2 roofline where the streamed weights fit in L2: read bandwidth of an
+    # L2-resident buffer of the same size, measured on the spot
+    l2_roof = None
+    if info.streamed_bytes <= 0.6 * props.L2_cache_size:
+        buf = torch.empty(info.streamed_bytes // 4, dtype=torch.float32, device="cuda")
+        buf.normal_()
+        with torch.cuda.stream(stream):
+            for _ in range(20):
+                buf.sum()
+            q0, q1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            q0.record(stream)
+            reps = 200
+            for _ in range(reps):
+                buf.sum()
+            q1.record(stream)
+        stream.synchronize()
+        l2_gbs = info.streamed_bytes * reps / (q0.elapsed_time(q1) * 1e-3) / 1e9
+        del buf
+        l2_roof = {"peak": l2_gbs, "unit": "GB/s", "frac": achieved / l2_gbs,
+                   "probe": f"torch sum over one {info.streamed_bytes / 1e6:.1f} MB float32 "
+                            f"buffer kept in L2 ({reps} back-to-back reads, CUDA events)"}
+
+    # end to end through the public API: token(s) in, host logits out, host
+    # argmax, at the same positions as the timed launches
     e2e = None
     if not args.no_e2e:
         import torch as _t
         host_logits = _t.empty(B * cfg["vocab_size"], dtype=_t.float32, pin_memory=True).numpy()
         V = cfg["vocab_size"]
         k_e2e = min(args.steps, 2048)
-        first = [tok0] if B == 1 else BATCH_STARTS[:B]
+        ewins = timed_windows(seq, k_e2e, pos0)
+        estarts = window_starts(ewins, pos0, first, fill)
 
         def api_step(toks, p):
             if B == 1:
@@ -493,30 +608,41 @@ def main():
                 model.forward_batch(toks, p, host_logits)
             return [int(np.argmax(host_logits[b * V:(b + 1) * V])) for b in range(B)]
 
-        toks = list(first)
-        for p in range(pos0, pos0 + 8):
-            toks = api_step(toks, p)
+        toks = list(estarts[-1])
+        for i in range(min(8, ewins[-1][1])):
+            toks = api_step(toks, ewins[-1][0] + i)
         t0 = time.perf_counter()
-        toks, pos = list(first), pos0
-        for s_ in range(k_e2e):
-            toks = api_step(toks, pos)
-            pos += 1
-            if pos == pos0 + seq:
-                toks, pos = list(first), pos0
+        for (p, n), st in zip(ewins, estarts):
+            toks = list(st)
+            for i in range(n):
+                toks = api_step(toks, p + i)
         e2e_s = time.perf_counter() - t0
         e2e = {"value": world * B * k_e2e / e2e_s, "unit": "tokens/s",
                "h2d_bytes_per_step": 4 * B, "d2h_bytes_per_step": 4 * B * V,
+               "positions": positions_of(ewins),
                "note": ("tvl_forward" if B == 1 else "tvl_forward_batch") +
                        " per step: token(s) as launch arguments, logits to pinned host "
                        "memory, argmax on the host"}
 
-    cpu = None
+    cpu = cpu_pm = None
     if rank == 0 and not args.no_cpu_baseline and args.workload in ("110m", "tiny"):
-        rate, n, el = cpu_oracle_rate(cfg, blob, args.cpu_seconds,
-                                      8 if args.weights == "q8" else 0)
+        import oracle
+        wb = 8 if args.weights == "q8" else 0
+        rate, n, el = cpu_decode_rate(lambda: oracle.Model(cfg, blob, 32, weight_bits=wb), cfg,
+                                      args.cpu_seconds)
         cpu = {"value": rate, "unit": "tokens/s", "cores": 1, "kind": "oracle",
-               "sample": f"first {n} greedy steps of the workload from token 1 "
-                         f"({el:.1f} s, double accumulators, one thread)"}
+               "sample": f"first {n} greedy steps of the workload from token 1 ({el:.1f} s, "
+                         f"float accumulators: the paper's scalar baseline, one thread)"}
+        if wb == 0:
+            import baseline
+            rate, n, el = cpu_decode_rate(lambda: baseline.Model(cfg, blob), cfg,
+                                          args.cpu_seconds / 2)
+            cpu_pm = {"value": rate, "unit": "tokens/s", "cores": 1,
+                      "kind": ("paper method: NEON float32x4 GEMV with four accumulators and "
+                               "NEON RMSNorm" if baseline.has_neon() else
+                               "paper method in plain C (this host has no NEON)"),
+                      "sample": f"first {n} greedy steps of the workload from token 1 "
+                                f"({el:.1f} s, one thread)"}
 
     value = job_tokens_per_s(world, args.steps, el_ms) * B
     # board energy per token (paper's energy section reports mJ/token): the
@@ -526,6 +652,8 @@ def main():
         energy = {"power_w": clk["power_w"],
                   "mj_per_token": 1e3 * clk["power_w"] * (el_ms * 1e-3) / (args.steps * B),
                   "note": "nvidia-smi power.draw (board), median over the timed region"}
+    streamed_cfg = streamed_bytes_of(cfg, 8 if args.weights == "q8" else 0)
+    assert streamed_cfg == info.streamed_bytes, (streamed_cfg, info.streamed_bytes)
     line = {
         "metric": METRIC if B == 1 else METRIC_BATCH.format(b=B), "value": value,
         "unit": "tokens/s", "n_gpus": world,
@@ -535,14 +663,15 @@ def main():
                         if args.workload == "110m" and args.weights == "f32" and B == 1 else None),
         "dtype": "f32" if args.weights == "f32" else "f32 activations, int8 weight rows",
         "data": "synthetic (seeded N(0, 0.02) weights)",
-        "config": dict(workload_config(args.workload, cfg, B, info.streamed_bytes,
-                                       props.L2_cache_size), weights=args.weights),
+        "config": workload_config(args.workload, cfg, B, args.weights, positions_of(wins)),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "kernel": "decode_kernel", "peak_source": peak_src,
-                     "bytes_per_launch": bytes_launch, "steps_per_launch": n_typ,
-                     "launch_ms": launch_ms},
+                     "bytes_per_launch": bytes_launch, "bytes_timed": bytes_timed,
+                     "launches": len(per), "kernel_ms": kern_ms, "l2": l2_roof},
+        "full_sequence": full_seq,
         "cpu_baseline": cpu,
+        "cpu_baseline_paper_method": cpu_pm,
         "e2e": e2e,
         "gpu_launches": launches,
         "clocks": clk,
@@ -550,8 +679,8 @@ def main():
                             "p90": float(np.percentile(dts, 90)),
                             "p99": float(np.percentile(dts, 99)),
                             "max": float(np.max(dts)), "std": float(np.std(dts)),
-                            "source": "device timestamps at the end of each step of one "
-                                      "launch (tvl_step_times)"},
+                            "source": "device timestamps at the end of each step of the "
+                                      "whole-sequence launch (tvl_step_times)"},
         "energy": energy,
         "grid": info.grid, "ring_stages": info.ring_stages,
         "prefill": prefill,

@@ -238,6 +238,27 @@ tvl_status tvl_gemv_q4(const void* Wq4, const float* x, float* y, int32_t d_out,
 tvl_status tvl_gemv_noalloc(const float* W, const float* x, float* y, int32_t d_out,
                             int32_t d_in, void* stream);
 
+/* Error report of the standalone GEMV calls (tvl_gemv, tvl_gemv_noalloc,
+ * tvl_gemv_q8, tvl_gemv_q4), which queue their kernel and return without
+ * waiting. Every wait inside those kernels is bounded (one second); when one
+ * runs out — only a broken device can cause it — the kernel raises
+ * TVL_E_TIMEOUT in an error word of the current device and its CTAs leave, so
+ * that call's y is incomplete. This call waits for the work queued on
+ * `stream`, then returns that error (and clears it) or TVL_OK. Split-K
+ * counters are tagged with their call, so calls after a failed one are
+ * correct whether or not this is called. Allocates nothing. */
+tvl_status tvl_gemv_status(void* stream);
+
+/* Failure-detection self-test of the standalone GEMV kernel: tvl_gemv_noalloc's
+ * kernel (same shape rules, same static scratch) runs with the last stage of
+ * CTA 0 never copied, so that CTA's consumer waits for it until the one-second
+ * limit runs out. Returns what tvl_gemv_status then reports: TVL_E_TIMEOUT
+ * expected, with the CUDA context still usable; y is left partly written.
+ * W, x, y as for tvl_gemv (a shape the streaming kernel takes, else
+ * TVL_E_UNSUPPORTED). */
+tvl_status tvl_selftest_gemv_timeout(const float* W, const float* x, float* y, int32_t d_out,
+                                     int32_t d_in, void* stream);
+
 /* Wait for the model's queued work, then report any device-side error. */
 tvl_status tvl_sync(tvl_model* m);
 
@@ -258,8 +279,9 @@ typedef struct {
   int32_t ring_stages;       /* weight staging ring: stages x stage_bytes */
   int32_t stage_bytes;
   int32_t tied;
-  int32_t barriers_per_step; /* grid-wide barriers in one greedy step */
-  int32_t max_batch;         /* as loaded (1 when the config said 0) */
+  int32_t exchanges_per_step; /* tagged exchanges between CTAs in one greedy step */
+  int32_t max_batch;          /* as loaded (1 when the config said 0) */
+  int64_t next_tag;           /* exchange tag the next launch starts from (1 .. 2^32 - 1) */
 } tvl_model_info;
 tvl_status tvl_get_info(const tvl_model* m, tvl_model_info* out);
 
@@ -267,11 +289,34 @@ tvl_status tvl_get_info(const tvl_model* m, tvl_model_info* out);
  * last tvl_decode_greedy call, for per-step latency statistics (§7.3). */
 tvl_status tvl_step_times(tvl_model* m, uint64_t* ns_out, int32_t n);
 
-/* Failure-detection self-test: launches the grid barrier of the decode kernel
- * against a count that nothing will reach, with a wait limit of limit_ms.
- * Expected result TVL_E_TIMEOUT, reported by the kernel itself, with the CUDA
- * context still usable. Uses the current device. */
+/* Failure-detection self-test: the decode kernel's bounded exchange poll
+ * (the consumer warps of one CTA polling a tagged word) waits on a word that
+ * nothing writes, with a wait limit of limit_ms (1 .. 10000). Expected result
+ * TVL_E_TIMEOUT, raised by the kernel itself, with the CUDA context still
+ * usable. Uses the current device. */
 tvl_status tvl_selftest_barrier_timeout(int32_t limit_ms);
+
+/* ---- Test hooks: not needed for normal use ---------------------------------
+ * They reach states that are otherwise hours of decoding or an out-of-memory
+ * device away. The paper has no counterpart. */
+
+/* Makes the k-th device or pinned-host allocation attempt of the library from
+ * now on fail as if memory were exhausted (k = 0: the next attempt); k < 0
+ * disarms. It fires once. Lets a test reach every failure point of tvl_load,
+ * tvl_prefill and tvl_gemv, which must then return TVL_E_NOMEM and hold no
+ * allocation. Process-wide; not thread-safe against concurrent loads. */
+void tvl_debug_fail_allocation(int32_t k);
+
+/* Device and pinned-host allocations the library holds right now (arenas,
+ * prefill activations, GEMV scratch buffers). */
+int64_t tvl_debug_live_allocations(void);
+
+/* Sets the exchange tag the model's next launch starts from (tvl_model_info.
+ * next_tag), 1 .. 2^32 - 1, else TVL_E_INVAL. Tags are 32-bit and 0 marks a
+ * word never written: a launch whose tags would pass 2^32 - 1 first zeroes
+ * the exchange words on the model's stream and starts again from tag 1. This
+ * hook puts a model next to that point without 2^32 exchanges of decoding. */
+tvl_status tvl_debug_set_next_tag(tvl_model* m, uint64_t tag);
 
 #ifdef __cplusplus
 }

@@ -1,4 +1,5 @@
 // abi.cu — status strings, per-thread error messages, blob layout and size.
+#include <atomic>
 #include <cstdio>
 #include <string>
 
@@ -7,6 +8,46 @@
 namespace tvl {
 
 static thread_local std::string g_last_error;
+
+// Allocation accounting and the failure injector (test hooks of include/tvl.h).
+static std::atomic<long long> g_live_allocs{0};
+static std::atomic<int> g_fail_countdown{-1};  // < 0: off; k: fail the k-th attempt from now
+
+static bool injected_failure() {
+  int k = g_fail_countdown.load();
+  while (k >= 0) {
+    if (g_fail_countdown.compare_exchange_weak(k, k - 1)) return k == 0;
+  }
+  return false;
+}
+
+cudaError_t lib_malloc(void** p, size_t bytes) {
+  *p = nullptr;
+  if (injected_failure()) return cudaErrorMemoryAllocation;
+  const cudaError_t e = cudaMalloc(p, bytes);
+  if (e == cudaSuccess) ++g_live_allocs;
+  return e;
+}
+
+void lib_free(void* p) {
+  if (!p) return;
+  cudaFree(p);
+  --g_live_allocs;
+}
+
+cudaError_t lib_host_alloc(void** p, size_t bytes, unsigned flags) {
+  *p = nullptr;
+  if (injected_failure()) return cudaErrorMemoryAllocation;
+  const cudaError_t e = cudaHostAlloc(p, bytes, flags);
+  if (e == cudaSuccess) ++g_live_allocs;
+  return e;
+}
+
+void lib_free_host(void* p) {
+  if (!p) return;
+  cudaFreeHost(p);
+  --g_live_allocs;
+}
 
 void set_error(const std::string& msg) { g_last_error = msg; }
 
@@ -94,5 +135,9 @@ const char* tvl_status_string(tvl_status s) {
 }
 
 const char* tvl_last_error(void) { return tvl::g_last_error.c_str(); }
+
+void tvl_debug_fail_allocation(int32_t k) { tvl::g_fail_countdown.store(k < 0 ? -1 : k); }
+
+int64_t tvl_debug_live_allocations(void) { return (int64_t)tvl::g_live_allocs.load(); }
 
 }  // extern "C"

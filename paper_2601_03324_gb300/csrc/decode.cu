@@ -97,8 +97,8 @@ tvl_status check_device_error(tvl_model* m) {
 void destroy(tvl_model* m) {
   if (!m) return;
   prefill_release(m);
-  if (m->arena) cudaFree(m->arena);
-  if (m->err_host) cudaFreeHost(m->err_host);
+  lib_free(m->arena);
+  lib_free_host(m->err_host);
   if (m->own_stream && m->stream) cudaStreamDestroy(m->stream);
   delete m;
 }
@@ -133,7 +133,18 @@ tvl_status launch(tvl_model* m, int B, const int* tokens, int pos, int n_steps,
   a.start_pos = pos;
   a.n_steps = n_steps;
   a.final_token = final_token;
-  a.epoch0 = m->epoch;
+  // Every exchange of the launch has its own tag; a tag must not repeat while
+  // a word may still hold it, and 0 marks a word never written.
+  const uint64_t span = (uint64_t)n_steps * (uint64_t)(kPhasesPerLayer * m->cfg.n_layers + 1);
+  if (span >= 0xFFFFFFFFull) {
+    set_error("launch: too many exchanges in one launch for 32-bit tags");
+    return TVL_E_RANGE;
+  }
+  if (m->next_tag + span > 0xFFFFFFFFull) {
+    TVL_CK(cudaMemsetAsync(m->arena + m->xchg_off, 0, m->xchg_bytes, m->stream));
+    m->next_tag = 1;
+  }
+  a.epoch0 = (unsigned)m->next_tag;
   const tvl_model::Plan& pl = m->plan[B];
   a.nst = pl.nst;
   a.sm_ring = pl.sm_ring; a.sm_bars = pl.sm_bars; a.sm_xs = pl.sm_xs; a.sm_vec = pl.sm_vec;
@@ -142,8 +153,7 @@ tvl_status launch(tvl_model* m, int B, const int* tokens, int pos, int n_steps,
   void* params[] = {&a};
   TVL_CK(cudaLaunchCooperativeKernel(m->kernel[B], dim3(a.G), dim3(kThreads), params,
                                      (size_t)pl.total, m->stream));
-  // tags wrap modulo 2^32; a stale word is never within one launch of a live tag
-  m->epoch += (unsigned)n_steps * (unsigned)(kPhasesPerLayer * m->cfg.n_layers + 1);
+  m->next_tag += span;
   return TVL_OK;
 }
 
@@ -308,7 +318,9 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   const size_t o_ts = take(8ull * S), o_err = take(4);
   m->arena_bytes = off;
   m->weight_bytes = blob_bytes;
-  if ((st = ck(cudaMalloc((void**)&m->arena, m->arena_bytes), "cudaMalloc(arena)")) != TVL_OK)
+  m->xchg_off = o_qkv;
+  m->xchg_bytes = o_tok - o_qkv;
+  if ((st = ck(lib_malloc((void**)&m->arena, m->arena_bytes), "cudaMalloc(arena)")) != TVL_OK)
     return fail(st);
   if (stream) {
     m->stream = (cudaStream_t)stream;
@@ -318,7 +330,7 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
       return fail(st);
     m->own_stream = true;
   }
-  if ((st = ck(cudaHostAlloc((void**)&m->err_host, sizeof(int), cudaHostAllocMapped),
+  if ((st = ck(lib_host_alloc((void**)&m->err_host, sizeof(int), cudaHostAllocMapped),
                "cudaHostAlloc(err)")) != TVL_OK)
     return fail(st);
   *m->err_host = 0;
@@ -375,7 +387,7 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   {  // the streamed [W1 | W3] blocks get interleaved rows
     const size_t row_bytes = q8 ? rq : 4ull * d;
     unsigned char* tmp = nullptr;
-    if (L > 0 && (st = ck(cudaMalloc((void**)&tmp, 2 * (size_t)F * row_bytes),
+    if (L > 0 && (st = ck(lib_malloc((void**)&tmp, 2 * (size_t)F * row_bytes),
                           "cudaMalloc(w13 scratch)")) != TVL_OK)
       return fail(st);
     for (int l = 0; l < L && st == TVL_OK; ++l) {
@@ -384,7 +396,7 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
       st = interleave_w13(blk, (size_t)F, row_bytes, tmp, m->stream);
     }
     if (st == TVL_OK) st = ck(cudaStreamSynchronize(m->stream), "cudaStreamSynchronize(w13)");
-    if (tmp) cudaFree(tmp);
+    lib_free(tmp);
     if (st != TVL_OK) return fail(st);
   }
 
@@ -605,7 +617,8 @@ tvl_status tvl_get_info(const tvl_model* m, tvl_model_info* out) {
   out->ring_stages = m->plan[1].nst;
   out->stage_bytes = kStageBytes;
   out->tied = m->tied ? 1 : 0;
-  out->barriers_per_step = kPhasesPerLayer * m->cfg.n_layers + 1;
+  out->exchanges_per_step = kPhasesPerLayer * m->cfg.n_layers + 1;
+  out->next_tag = (int64_t)m->next_tag;
   out->max_batch = m->max_batch;
   return TVL_OK;
 }
@@ -620,13 +633,22 @@ tvl_status tvl_step_times(tvl_model* m, uint64_t* ns_out, int32_t n) {
   return TVL_OK;
 }
 
+tvl_status tvl_debug_set_next_tag(tvl_model* m, uint64_t tag) {
+  if (!m || tag < 1 || tag > 0xFFFFFFFFull) {
+    set_error("tvl_debug_set_next_tag: null model or tag outside [1, 2^32 - 1]");
+    return TVL_E_INVAL;
+  }
+  m->next_tag = tag;
+  return TVL_OK;
+}
+
 tvl_status tvl_selftest_barrier_timeout(int32_t limit_ms) {
   if (limit_ms < 1 || limit_ms > 10000) {
     set_error("tvl_selftest_barrier_timeout: limit_ms out of [1, 10000]");
     return TVL_E_INVAL;
   }
   unsigned char* buf = nullptr;
-  TVL_CK(cudaMalloc((void**)&buf, 256));
+  TVL_CK(lib_malloc((void**)&buf, 256));
   tvl_status st = TVL_OK;
   cudaError_t e = cudaMemset(buf, 0, 256);  // tag 0: never the awaited tag 1
   if (e == cudaSuccess) {
@@ -639,7 +661,7 @@ tvl_status tvl_selftest_barrier_timeout(int32_t limit_ms) {
   int code = 0;
   if (e == cudaSuccess) e = cudaMemcpy(&code, buf + 64, sizeof(int), cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) st = cuda_fail(e, "wait self-test");
-  cudaFree(buf);
+  lib_free(buf);
   if (st != TVL_OK) return st;
   if (code == 0) {
     set_error("wait self-test: the wait did not report a timeout");

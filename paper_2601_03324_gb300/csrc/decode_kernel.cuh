@@ -491,6 +491,16 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
     const int gi = tid / hd4, f = tid - gi * hd4;
     const int n = t1 - t0;
     const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
+    // this thread's q/k/v pair (at most one: nget <= 3 hd / 2 <= 192 < 224
+    // threads) is asked for first, so that its poll is not queued behind the
+    // row loads below
+    const int nget = has_new ? 3 * half : half;
+    const int tq = tid < nget ? tid : 0;  // head_dim <= 128 keeps nget below 224
+    const int which0 = tq / half, i0 = tq - which0 * half;
+    const unsigned long long* src0 =
+        xq + (which0 == 0 ? h * hd : a.d + (which0 - 1) * a.kvd + kvh * hd) + 2 * i0;
+    ulonglong2 qv = make_ulonglong2(0ull, 0ull);
+    if (tid < nget) qv = ld_tag2(src0);
     // the first three K and V rows of each thread, loaded before q is ready
     float4 kr0 = z4, kr1 = z4, kr2 = z4, v0 = z4, v1 = z4, v2 = z4;
     {
@@ -511,14 +521,20 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
     }
     // q (and the new k, v) with RoPE: pair i turns by pos * theta^(-2i/hd).
     // Pair i of a head is one 16-byte tagged load.
-    const int nget = has_new ? 3 * half : half;
     bool ok = true;
-    for (int t = tid; t < nget && ok; t += kConsumerThreads) {
-      const int which = t / half, i = t - which * half;
-      const unsigned long long* src =
-          xq + (which == 0 ? h * hd : a.d + (which - 1) * a.kvd + kvh * hd) + 2 * i;
-      ulonglong2 v;
-      ok = poll_one(src, tag_qkv, pc, v);
+    if (tid < nget) {
+      const int which = which0, i = i0;
+      ulonglong2 v = qv;
+      {
+        PollClock clk;
+        while (!tags_are(v, tag_qkv)) {
+          if (!clk.keep_waiting(pc)) {
+            ok = false;
+            break;
+          }
+          v = ld_tag2(src0);
+        }
+      }
       const float x0 = lo_f(v.x), x1 = lo_f(v.y);
       if (which == 2) {
         vp[2 * i] = x0;
@@ -784,7 +800,7 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
   constexpr int kPollDepthH = kB == 1 ? 5 : 8;
   const Poll pc{a.err, a.err_host, s_abort, a.wait_limit_ns};
   const unsigned per_step = (unsigned)(kPhasesPerLayer * a.L + 1);
-  uint32_t g = 0;
+  StageCursor cur;
   int token[kB];
 #pragma unroll
   for (int b = 0; b < kB; ++b) token[b] = a.start_tokens[b];
@@ -938,11 +954,13 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
         EpiTag e{out, el + (k == 0 ? 0u : (unsigned)k + 1u), k == 2 ? a.F : M, k == 2,
                  {rs[0], rs[1], rs[2], rs[3]}};
         if constexpr (kQ8) {
+          uint32_t g = cur.g;
           if (!consume_phase<false, kQ8>(r, g, plan, vec, 1, K, seg, e, a.err, a.err_host,
                                          s_abort))
             return false;
+          cur.advance(plan.nstages, r.nst);
         } else {
-          if (!consume_phase_b<kB>(r, g, plan, vec, vs, seg, e, a.err, a.err_host, s_abort))
+          if (!consume_phase_b<kB>(r, cur, plan, vec, vs, seg, e, a.err, a.err_host, s_abort))
             return false;
         }
       }
@@ -960,11 +978,13 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
     EpiArgmax<kB> ea{a.logits, a.V, {rs[0], rs[1], rs[2], rs[3]}};
     ea.init();
     if constexpr (kQ8) {
+      uint32_t g = cur.g;
       if (!consume_phase<false, kQ8>(r, g, plans[4], vec, 1, a.d, seg, ea, a.err, a.err_host,
                                      s_abort))
         return false;
+      cur.advance(plans[4].nstages, r.nst);
     } else {
-      if (!consume_phase_b<kB>(r, g, plans[4], vec, vs, seg, ea, a.err, a.err_host, s_abort))
+      if (!consume_phase_b<kB>(r, cur, plans[4], vec, vs, seg, ea, a.err, a.err_host, s_abort))
         return false;
     }
 #pragma unroll

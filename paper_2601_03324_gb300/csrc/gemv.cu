@@ -1,17 +1,21 @@
 // gemv.cu — standalone y = W x (paper §6.1) on the weight-streaming engine.
 //
 // One CTA per SM streams its contiguous share of W through the shared-memory
-// stage ring (a producer warp and seven consumer warps). Matrices with few rows are split along K into S chunks so that
-// every SM gets work: virtual row v = (row v / S, chunk v % S); each virtual
-// row's partial lands in a scratch buffer, and each row is summed over its
-// S chunks in chunk order — by the CTA that owns the whole row, or for a row
-// shared by two CTAs, by whichever of them finishes last (a per-row arrival
-// counter). The result does not depend on timing. Every wait in the kernel is
-// bounded (one second); a CTA whose stage never lands leaves early, which
-// only a broken device can cause.
+// stage ring (a producer warp and seven consumer warps). Matrices with few
+// rows are split along K into S chunks so that every SM gets work: virtual
+// row v = (row v / S, chunk v % S); each virtual row's partial lands in a
+// scratch buffer, and each row is summed over its S chunks in chunk order — by
+// the CTA that owns the whole row, or for a row shared by two CTAs, by
+// whichever of them finishes last (a per-row arrival counter tagged with the
+// call's id, so that a call that gave up part-way leaves nothing the next
+// call would count). The result does not depend on timing. Every wait in the
+// kernel is bounded (one second); a CTA whose stage never lands raises
+// TVL_E_TIMEOUT in the module's error word (tvl_gemv_status reports it) and
+// leaves early, which only a broken device can cause.
 #include <cstdio>
 #include <map>
 #include <mutex>
+#include <string>
 #include <utility>
 
 #include "host_common.h"
@@ -28,7 +32,10 @@ struct GemvArgs {
   int M, K, S, Kc;
   long long nv;  // virtual rows = M * S
   float* part;   // [M * S] when S > 1
-  int* cnt;      // [M], zero between calls
+  unsigned* cnt; // [M]: (call id << 8) | chunks counted, for the call that last touched the row
+  unsigned call_id;  // 1 .. 2^24 - 1, different for consecutive calls sharing cnt
+  int* err;          // the module's error word (TVL_E_TIMEOUT after a wait ran out)
+  int drop_last;     // self-test: CTA 0's producer never copies its last stage
   int nst;
   int sm_ring, sm_bars, sm_x, sm_seg, sm_misc;
 };
@@ -82,7 +89,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   if (threadIdx.x >= kConsumerThreads) {
     if (threadIdx.x == kConsumerThreads) {
       GemvSched sched{a.W, 0u, p, false};
-      run_producer(r, sched, nullptr, nullptr, s_abort);
+      if (a.drop_last && blockIdx.x == 0 && sched.p.nstages > 0) --sched.p.nstages;
+      run_producer(r, sched, a.err, nullptr, s_abort);
     }
     return;
   }
@@ -94,30 +102,44 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   named_bar_sync(kBarConsumers, kConsumerThreads);
   if (a.S == 1) {
     EpiStore e{a.y};
-    consume_phase<true, kQ8, kQ4>(r, g, p, xs, 1, a.Kc, seg, e, nullptr, nullptr, s_abort);
+    consume_phase<true, kQ8, kQ4>(r, g, p, xs, 1, a.Kc, seg, e, a.err, nullptr, s_abort);
     return;
   }
   EpiPart e{a.part};
-  if (!consume_phase(r, g, p, xs, a.S, a.Kc, seg, e, nullptr, nullptr, s_abort)) return;
+  if (!consume_phase(r, g, p, xs, a.S, a.Kc, seg, e, a.err, nullptr, s_abort)) return;
   if (p.r1 <= p.r0) return;
   named_bar_sync(kBarConsumers, kConsumerThreads);
   const int S = a.S;
   const int ra = p.r0 / S, rb = (p.r1 - 1) / S;
+  const unsigned id = a.call_id << 8;
   for (int row = ra + threadIdx.x; row <= rb; row += kConsumerThreads) {
     const int lo = max(p.r0, row * S), hi = min(p.r1, (row + 1) * S);
-    const int mine = hi - lo;
-    bool last = (mine == S);
+    const unsigned mine = (unsigned)(hi - lo);
+    bool last = (mine == (unsigned)S);
     if (!last) {
+      // add this CTA's chunks to the row's count for this call; a count left
+      // by another call (one that gave up part-way) counts as zero
       __threadfence();
-      const int before = atomicAdd(a.cnt + row, mine);
-      last = (before + mine == S);
+      unsigned* c = a.cnt + row;
+      unsigned old = *reinterpret_cast<volatile unsigned*>(c), before = 0;
+      bool added = false;
+      for (int it = 0; it < (1 << 16) && !added; ++it) {
+        before = (old & ~0xFFu) == id ? (old & 0xFFu) : 0u;
+        const unsigned seen = atomicCAS(c, old, id | (before + mine));
+        added = seen == old;
+        old = seen;
+      }
+      if (!added) {  // cannot happen while calls sharing cnt are ordered
+        raise_error(a.err, nullptr, kErrTimeout);
+        continue;
+      }
+      last = (before + mine == (unsigned)S);
       if (last) __threadfence();
     }
     if (last) {
       float v = 0.f;
       for (int s = 0; s < S; ++s) v += __ldcg(a.part + (size_t)row * S + s);
       a.y[row] = v;
-      if (mine != S) a.cnt[row] = 0;
     }
   }
 }
@@ -206,27 +228,122 @@ __global__ void quantize_q4_kernel(const float* __restrict__ W, unsigned char* _
 
 namespace {
 
-struct Workspace {
-  float* part = nullptr;
-  int* cnt = nullptr;
-  long long part_cap = 0;
-  int cnt_cap = 0;
-};
-
-std::mutex g_ws_mu;
-std::map<std::pair<int, cudaStream_t>, Workspace> g_ws;
+// The module's error word: every standalone GEMV kernel raises a timeout
+// here; tvl_gemv_status reads and clears it. One per device.
+static __device__ int g_gemv_err;
 
 struct DevInfo {
   int sms = 0, max_optin = 0;
-  bool attr_set = false;
+  int* err = nullptr;  // device address of g_gemv_err on this device
 };
-std::map<int, DevInfo> g_dev;
+std::mutex g_dev_mu;
+constexpr int kMaxDevices = 64;
+DevInfo g_dev[kMaxDevices];  // fixed table: no heap use on any call
+
+// Attributes of the current device and the address of its error word
+// (looked up once per device).
+tvl_status dev_info(const char* who, DevInfo* out) {
+  int dev = 0;
+  TVL_CK(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kMaxDevices) {
+    char msg[160];
+    snprintf(msg, sizeof msg, "%s: device ordinal %d is beyond the %d-entry table", who, dev,
+             kMaxDevices);
+    set_error(msg);
+    return TVL_E_UNSUPPORTED;
+  }
+  std::lock_guard<std::mutex> lk(g_dev_mu);
+  DevInfo& di = g_dev[dev];
+  if (di.sms == 0) {
+    void* e = nullptr;
+    TVL_CK(cudaGetSymbolAddress(&e, g_gemv_err));
+    TVL_CK(cudaDeviceGetAttribute(&di.max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev));
+    int sms = 0;
+    TVL_CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    di.err = reinterpret_cast<int*>(e);
+    di.sms = sms;
+  }
+  *out = di;
+  return TVL_OK;
+}
+
+// The next call id of a counter set (1 .. 2^24 - 1, never 0: zeroed counters
+// belong to no call).
+unsigned next_call_id(unsigned* next) {
+  const unsigned id = *next;
+  *next = id >= 0xFFFFFFu ? 1u : id + 1u;
+  return id;
+}
 
 int split_for(int M, int K, int G) {
   int S = 1;
   while ((long long)M * S < 16LL * G && K % (8 * S) == 0 && K / (2 * S) >= 128) S *= 2;
   return S;
 }
+
+// Whether the streaming kernel takes W [M x K] (else the per-row kernel):
+// 16-byte aligned W and x, K % 4 == 0, K <= 16384, and the segment partials
+// of rows longer than a stage fit the shared scratch.
+bool streams(const float* W, const float* x, int M, int K, int sms, int* S_out) {
+  const bool aligned = ((uintptr_t)W % 16 == 0) && ((uintptr_t)x % 16 == 0) && K % 4 == 0;
+  if (!aligned || K > 16384) return false;
+  const int S = split_for(M, K, sms);
+  const long long nv = (long long)M * S;
+  const long long G = nv < sms ? nv : sms;
+  const StagePlan pl = plan_stages(nv, K / S, (int)G, 0);
+  *S_out = S;
+  return pl.spr == 1 || ((nv + G - 1) / G) * pl.spr <= kMaxSegParts;
+}
+
+tvl_status launch_rowwise(const float* W, const float* x, float* y, int M, int K,
+                          cudaStream_t s) {
+  const int threads = 256, rows_per_block = threads / 32;
+  gemv_rowwise_kernel<<<(M + rows_per_block - 1) / rows_per_block, threads, 0, s>>>(W, x, y, M,
+                                                                                     K);
+  TVL_CK(cudaGetLastError());
+  return TVL_OK;
+}
+
+// Shared memory (ring | barriers | x | segment partials | misc, every region a
+// 128-byte multiple) and launch of gemv_stream_kernel<kQ8, kQ4> for a.nv
+// virtual rows of a.Kc words; a.K floats of x.
+template <bool kQ8, bool kQ4>
+tvl_status launch_stream(GemvArgs& a, const DevInfo& di, cudaStream_t s, const char* who) {
+  const int G = (int)(a.nv < di.sms ? a.nv : di.sms);
+  const int xbytes = (int)a128(4LL * a.K), segb = (int)a128(kMaxSegParts * 4);
+  const int bars = (int)a128(kRingBarBytes);
+  const int misc = 128;
+  int nst = (di.max_optin - xbytes - segb - bars - misc) / kStageBytes;
+  if (nst > kMaxStages) nst = kMaxStages;
+  if (nst < 2) {
+    set_error(std::string(who) + ": not enough shared memory");
+    return TVL_E_UNSUPPORTED;
+  }
+  a.err = di.err;
+  a.nst = nst;
+  a.sm_ring = 0;
+  a.sm_bars = nst * kStageBytes;
+  a.sm_x = a.sm_bars + bars;
+  a.sm_seg = a.sm_x + xbytes;
+  a.sm_misc = a.sm_seg + segb;
+  const int smem = a.sm_misc + misc;
+  TVL_CK(cudaFuncSetAttribute((const void*)gemv_stream_kernel<kQ8, kQ4>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+  gemv_stream_kernel<kQ8, kQ4><<<G, kThreads, smem, s>>>(a);
+  TVL_CK(cudaGetLastError());
+  return TVL_OK;
+}
+
+// Per-stream split-K scratch of tvl_gemv, allocated on first use.
+struct Workspace {
+  float* part = nullptr;
+  unsigned* cnt = nullptr;
+  long long part_cap = 0;
+  int cnt_cap = 0;
+  unsigned next_id = 1;
+};
+std::mutex g_ws_mu;
+std::map<std::pair<int, cudaStream_t>, Workspace> g_ws;
 
 }  // namespace
 
@@ -237,113 +354,136 @@ extern "C" tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t
     return TVL_E_INVAL;
   }
   cudaStream_t s = (cudaStream_t)stream;
-  int dev = 0;
-  TVL_CK(cudaGetDevice(&dev));
-  DevInfo info;
-  {
-    std::lock_guard<std::mutex> lk(g_ws_mu);
-    DevInfo& di = g_dev[dev];
-    if (di.sms == 0) {
-      cudaDeviceGetAttribute(&di.sms, cudaDevAttrMultiProcessorCount, dev);
-      cudaDeviceGetAttribute(&di.max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-    }
-    info = di;
-  }
-  const bool aligned = ((uintptr_t)W % 16 == 0) && ((uintptr_t)x % 16 == 0) && d_in % 4 == 0;
-  bool fits = aligned && d_in <= 16384;
-  if (fits) {  // segment partials of rows longer than a stage must fit the scratch
-    const int S = split_for(d_out, d_in, info.sms);
-    const long long nv = (long long)d_out * S;
-    const StagePlan pl = plan_stages(nv, d_in / S, (int)(nv < info.sms ? nv : info.sms), 0);
-    const long long G = nv < info.sms ? nv : info.sms;
-    fits = pl.spr == 1 || ((nv + G - 1) / G) * pl.spr <= kMaxSegParts;
-  }
-  if (!fits) {
-    const int threads = 256, rows_per_block = threads / 32;
-    gemv_rowwise_kernel<<<(d_out + rows_per_block - 1) / rows_per_block, threads, 0, s>>>(
-        W, x, y, d_out, d_in);
-    TVL_CK(cudaGetLastError());
-    return TVL_OK;
-  }
+  DevInfo di;
+  tvl_status st = dev_info("tvl_gemv", &di);
+  if (st != TVL_OK) return st;
+  int S = 1;
+  if (!streams(W, x, d_out, d_in, di.sms, &S)) return launch_rowwise(W, x, y, d_out, d_in, s);
   GemvArgs a{};
   a.W = W;
   a.x = x;
   a.y = y;
   a.M = d_out;
   a.K = d_in;
-  a.S = split_for(d_out, d_in, info.sms);
-  a.Kc = d_in / a.S;
-  a.nv = (long long)d_out * a.S;
-  const int G = (int)(a.nv < info.sms ? a.nv : info.sms);
-  // shared memory: ring | barriers | x | piece sums | misc
-  const int xbytes = (int)a128(4LL * d_in), segb = (int)a128(kMaxSegParts * 4);
-  const int bars = (int)a128(kRingBarBytes);  // every region a 128-byte multiple
-  const int misc = 128;
-  int nst = (info.max_optin - xbytes - segb - bars - misc) / kStageBytes;
-  if (nst > kMaxStages) nst = kMaxStages;
-  if (nst < 2) {
-    set_error("tvl_gemv: not enough shared memory");
-    return TVL_E_UNSUPPORTED;
-  }
-  a.nst = nst;
-  a.sm_ring = 0;
-  a.sm_bars = nst * kStageBytes;
-  a.sm_x = a.sm_bars + bars;
-  a.sm_seg = a.sm_x + xbytes;
-  a.sm_misc = a.sm_seg + segb;
-  const int smem = a.sm_misc + misc;
-  {
+  a.S = S;
+  a.Kc = d_in / S;
+  a.nv = (long long)d_out * S;
+  if (S > 1) {
+    int dev = 0;
+    TVL_CK(cudaGetDevice(&dev));
     std::lock_guard<std::mutex> lk(g_ws_mu);
     Workspace& ws = g_ws[{dev, s}];
-    const long long need_part = a.S > 1 ? a.nv : 1;
-    const int need_cnt = a.S > 1 ? d_out : 1;
-    if (ws.part_cap < need_part || ws.cnt_cap < need_cnt || !ws.part) {
-      if (ws.part) {  // earlier kernels on this stream may still use the old buffers
+    if (ws.part_cap < a.nv || ws.cnt_cap < d_out) {
+      if (ws.part || ws.cnt) {  // earlier kernels on this stream may still use the old buffers
         TVL_CK(cudaStreamSynchronize(s));
-        cudaFree(ws.part);
-        cudaFree(ws.cnt);
-        ws = Workspace{};
+        lib_free(ws.part);
+        lib_free(ws.cnt);
+        ws.part = nullptr;
+        ws.cnt = nullptr;
+        ws.part_cap = ws.cnt_cap = 0;
       }
-      const long long pc = need_part > 4096 ? need_part : 4096;
-      const int cc = need_cnt > 4096 ? need_cnt : 4096;
-      TVL_CK(cudaMalloc((void**)&ws.part, 4 * pc + 256));
-      TVL_CK(cudaMalloc((void**)&ws.cnt, 4LL * cc + 256));
-      TVL_CK(cudaMemsetAsync(ws.cnt, 0, 4LL * cc + 256, s));
+      const long long pc = a.nv > 4096 ? a.nv : 4096;
+      const int cc = d_out > 4096 ? d_out : 4096;
+      cudaError_t e = lib_malloc((void**)&ws.part, 4 * pc + 256);
+      if (e == cudaSuccess) e = lib_malloc((void**)&ws.cnt, 4LL * cc + 256);
+      if (e == cudaSuccess) e = cudaMemsetAsync(ws.cnt, 0, 4LL * cc + 256, s);
+      if (e != cudaSuccess) {
+        lib_free(ws.part);
+        lib_free(ws.cnt);
+        ws.part = nullptr;
+        ws.cnt = nullptr;
+        return cuda_fail(e, "tvl_gemv: split-K scratch");
+      }
       ws.part_cap = pc;
       ws.cnt_cap = cc;
     }
     a.part = ws.part;
     a.cnt = ws.cnt;
+    a.call_id = next_call_id(&ws.next_id);
   }
-  TVL_CK(cudaFuncSetAttribute((const void*)gemv_stream_kernel<false>,
-                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-  gemv_stream_kernel<false><<<G, kThreads, smem, s>>>(a);
-  TVL_CK(cudaGetLastError());
-  return TVL_OK;
+  return launch_stream<false, false>(a, di, s, "tvl_gemv");
 }
 
 // ---- tvl_gemv_noalloc: the same GEMV with its split-K scratch in module memory ----
 
 namespace {
 
-// Split-K partials (floats) and per-row arrival counters (ints) of
-// tvl_gemv_noalloc. split_for keeps M * S below 32 x the SM count and M below
-// 16 x the SM count whenever S > 1, so on a 152-SM part at most 4864 partials
-// and 2431 counters are live; the sizes below leave room for larger parts.
+// Split-K partials (floats) and per-row arrival counters of tvl_gemv_noalloc.
+// split_for keeps M * S below 32 x the SM count and M below 16 x the SM count
+// whenever S > 1, so on a 152-SM part at most 4864 partials and 2431 counters
+// are live; the sizes below leave room for larger parts.
 constexpr int kNoAllocPart = 8192;
 constexpr int kNoAllocRows = 4096;
 constexpr size_t kNoAllocBytes = 4 * (size_t)kNoAllocPart + 4 * (size_t)kNoAllocRows;  // 48 KB
 static __device__ __align__(256) unsigned char g_gemv_scratch[kNoAllocBytes];
 
-constexpr int kNoAllocMaxDevices = 64;
 struct NoAllocDev {
   bool ready;
-  int sms, max_optin;
   float* part;
-  int* cnt;
+  unsigned* cnt;
+  unsigned next_id;
 };
-NoAllocDev g_noalloc[kNoAllocMaxDevices];  // fixed table: no heap use on any call
+NoAllocDev g_noalloc[kMaxDevices];  // fixed table: no heap use on any call
 std::mutex g_noalloc_mu;
+
+// The static scratch of the current device (device addresses; the first call
+// on a device looks them up and zeroes the counters on `s`, waiting for it),
+// and the call's id. drop_last: see tvl_selftest_gemv_timeout.
+tvl_status noalloc_gemv(const float* W, const float* x, float* y, int d_out, int d_in,
+                        cudaStream_t s, int drop_last, const char* who) {
+  DevInfo di;
+  tvl_status st = dev_info(who, &di);
+  if (st != TVL_OK) return st;
+  int dev = 0;
+  TVL_CK(cudaGetDevice(&dev));
+  int S = 1;
+  if (!streams(W, x, d_out, d_in, di.sms, &S)) {
+    if (drop_last) {
+      set_error(std::string(who) + ": the shape does not take the streaming kernel");
+      return TVL_E_UNSUPPORTED;
+    }
+    return launch_rowwise(W, x, y, d_out, d_in, s);
+  }
+  const long long nv = (long long)d_out * S;
+  if (S > 1 && (nv > kNoAllocPart || d_out > kNoAllocRows)) {
+    char msg[192];
+    snprintf(msg, sizeof msg,
+             "%s: %d x %d splits into %lld partials over %d rows; the static scratch holds %d "
+             "partials and %d rows (use tvl_gemv)",
+             who, d_out, d_in, nv, d_out, kNoAllocPart, kNoAllocRows);
+    set_error(msg);
+    return TVL_E_UNSUPPORTED;
+  }
+  GemvArgs a{};
+  {
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    NoAllocDev& e = g_noalloc[dev];
+    if (!e.ready) {  // once per device: address of the module array, counters to zero
+      void* base = nullptr;
+      TVL_CK(cudaGetSymbolAddress(&base, g_gemv_scratch));
+      e.part = reinterpret_cast<float*>(base);
+      e.cnt = reinterpret_cast<unsigned*>(reinterpret_cast<unsigned char*>(base) +
+                                          4 * (size_t)kNoAllocPart);
+      TVL_CK(cudaMemsetAsync(e.cnt, 0, 4 * (size_t)kNoAllocRows, s));
+      TVL_CK(cudaStreamSynchronize(s));
+      e.next_id = 1;
+      e.ready = true;
+    }
+    a.part = e.part;
+    a.cnt = e.cnt;
+    a.call_id = next_call_id(&e.next_id);
+  }
+  a.W = W;
+  a.x = x;
+  a.y = y;
+  a.M = d_out;
+  a.K = d_in;
+  a.S = S;
+  a.Kc = d_in / S;
+  a.nv = nv;
+  a.drop_last = drop_last;
+  return launch_stream<false, false>(a, di, s, who);
+}
 
 }  // namespace
 
@@ -353,91 +493,38 @@ extern "C" tvl_status tvl_gemv_noalloc(const float* W, const float* x, float* y,
     set_error("tvl_gemv_noalloc: null pointer or non-positive size");
     return TVL_E_INVAL;
   }
-  cudaStream_t s = (cudaStream_t)stream;
-  int dev = 0;
-  TVL_CK(cudaGetDevice(&dev));
-  if (dev < 0 || dev >= kNoAllocMaxDevices) {
-    char msg[128];
-    snprintf(msg, sizeof msg, "tvl_gemv_noalloc: device ordinal %d is beyond the %d-entry table",
-             dev, kNoAllocMaxDevices);
-    set_error(msg);
-    return TVL_E_UNSUPPORTED;
+  return noalloc_gemv(W, x, y, d_out, d_in, (cudaStream_t)stream, 0, "tvl_gemv_noalloc");
+}
+
+extern "C" tvl_status tvl_gemv_status(void* stream) {
+  DevInfo di;
+  tvl_status st = dev_info("tvl_gemv_status", &di);
+  if (st != TVL_OK) return st;
+  TVL_CK(cudaStreamSynchronize((cudaStream_t)stream));
+  int code = 0;
+  TVL_CK(cudaMemcpy(&code, di.err, sizeof(int), cudaMemcpyDeviceToHost));
+  if (code == 0) return TVL_OK;
+  TVL_CK(cudaMemset(di.err, 0, sizeof(int)));
+  set_error("a bounded wait in a standalone GEMV kernel expired; the outputs of that call are "
+            "incomplete");
+  return (tvl_status)code;
+}
+
+extern "C" tvl_status tvl_selftest_gemv_timeout(const float* W, const float* x, float* y,
+                                                int32_t d_out, int32_t d_in, void* stream) {
+  if (!W || !x || !y || d_out < 1 || d_in < 1) {
+    set_error("tvl_selftest_gemv_timeout: null pointer or non-positive size");
+    return TVL_E_INVAL;
   }
-  NoAllocDev nd;
-  {
-    std::lock_guard<std::mutex> lk(g_noalloc_mu);
-    NoAllocDev& e = g_noalloc[dev];
-    if (!e.ready) {  // once per device: address of the module array, counters to zero
-      void* base = nullptr;
-      TVL_CK(cudaGetSymbolAddress(&base, g_gemv_scratch));
-      TVL_CK(cudaDeviceGetAttribute(&e.sms, cudaDevAttrMultiProcessorCount, dev));
-      TVL_CK(cudaDeviceGetAttribute(&e.max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev));
-      e.part = reinterpret_cast<float*>(base);
-      e.cnt = reinterpret_cast<int*>(reinterpret_cast<unsigned char*>(base) + 4 * (size_t)kNoAllocPart);
-      TVL_CK(cudaMemsetAsync(e.cnt, 0, 4 * (size_t)kNoAllocRows, s));
-      TVL_CK(cudaStreamSynchronize(s));
-      e.ready = true;
-    }
-    nd = e;
+  tvl_status st = noalloc_gemv(W, x, y, d_out, d_in, (cudaStream_t)stream, 1,
+                               "tvl_selftest_gemv_timeout");
+  if (st != TVL_OK) return st;
+  st = tvl_gemv_status(stream);
+  if (st == TVL_OK) {
+    set_error("gemv self-test: the wait on the missing stage did not report a timeout");
+    return TVL_E_CUDA;
   }
-  const bool aligned = ((uintptr_t)W % 16 == 0) && ((uintptr_t)x % 16 == 0) && d_in % 4 == 0;
-  bool fits = aligned && d_in <= 16384;
-  const int S = fits ? split_for(d_out, d_in, nd.sms) : 1;
-  const long long nv = (long long)d_out * S;
-  if (fits) {  // segment partials of rows longer than a stage must fit the shared scratch
-    const long long G = nv < nd.sms ? nv : nd.sms;
-    const StagePlan pl = plan_stages(nv, d_in / S, (int)G, 0);
-    fits = pl.spr == 1 || ((nv + G - 1) / G) * pl.spr <= kMaxSegParts;
-  }
-  if (!fits) {
-    const int threads = 256, rows_per_block = threads / 32;
-    gemv_rowwise_kernel<<<(d_out + rows_per_block - 1) / rows_per_block, threads, 0, s>>>(
-        W, x, y, d_out, d_in);
-    TVL_CK(cudaGetLastError());
-    return TVL_OK;
-  }
-  if (S > 1 && (nv > kNoAllocPart || d_out > kNoAllocRows)) {
-    char msg[192];
-    snprintf(msg, sizeof msg,
-             "tvl_gemv_noalloc: %d x %d splits into %lld partials over %d rows; the static "
-             "scratch holds %d partials and %d rows (use tvl_gemv)",
-             (int)d_out, (int)d_in, nv, (int)d_out, kNoAllocPart, kNoAllocRows);
-    set_error(msg);
-    return TVL_E_UNSUPPORTED;
-  }
-  GemvArgs a{};
-  a.W = W;
-  a.x = x;
-  a.y = y;
-  a.M = d_out;
-  a.K = d_in;
-  a.S = S;
-  a.Kc = d_in / S;
-  a.nv = nv;
-  a.part = nd.part;
-  a.cnt = nd.cnt;
-  const int G = (int)(nv < nd.sms ? nv : nd.sms);
-  const int xbytes = (int)a128(4LL * d_in), segb = (int)a128(kMaxSegParts * 4);
-  const int bars = (int)a128(kRingBarBytes);
-  const int misc = 128;
-  int nst = (nd.max_optin - xbytes - segb - bars - misc) / kStageBytes;
-  if (nst > kMaxStages) nst = kMaxStages;
-  if (nst < 2) {
-    set_error("tvl_gemv_noalloc: not enough shared memory");
-    return TVL_E_UNSUPPORTED;
-  }
-  a.nst = nst;
-  a.sm_ring = 0;
-  a.sm_bars = nst * kStageBytes;
-  a.sm_x = a.sm_bars + bars;
-  a.sm_seg = a.sm_x + xbytes;
-  a.sm_misc = a.sm_seg + segb;
-  const int smem = a.sm_misc + misc;
-  TVL_CK(cudaFuncSetAttribute((const void*)gemv_stream_kernel<false>,
-                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-  gemv_stream_kernel<false><<<G, kThreads, smem, s>>>(a);
-  TVL_CK(cudaGetLastError());
-  return TVL_OK;
+  return st;
 }
 
 // ---- weight-only 8-bit rows: quantization and GEMV --------------------------------
@@ -479,11 +566,9 @@ extern "C" tvl_status tvl_gemv_q8(const void* Wq8, const float* x, float* y, int
     set_error("tvl_gemv_q8: a packed row must fit one 16 KB stage (d_in <= 16368)");
     return TVL_E_UNSUPPORTED;
   }
-  cudaStream_t s = (cudaStream_t)stream;
-  int dev = 0, sms = 0, max_optin = 0;
-  TVL_CK(cudaGetDevice(&dev));
-  TVL_CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-  TVL_CK(cudaDeviceGetAttribute(&max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev));
+  DevInfo di;
+  tvl_status st = dev_info("tvl_gemv_q8", &di);
+  if (st != TVL_OK) return st;
   GemvArgs a{};
   a.W = reinterpret_cast<const float*>(Wq8);
   a.x = x;
@@ -493,28 +578,7 @@ extern "C" tvl_status tvl_gemv_q8(const void* Wq8, const float* x, float* y, int
   a.S = 1;
   a.Kc = Kw;
   a.nv = d_out;
-  const int G = d_out < sms ? d_out : sms;
-  const int xbytes = (int)a128(4LL * d_in), segb = (int)a128(kMaxSegParts * 4);
-  const int bars = (int)a128(kRingBarBytes);
-  const int misc = 128;
-  int nst = (max_optin - xbytes - segb - bars - misc) / kStageBytes;
-  if (nst > kMaxStages) nst = kMaxStages;
-  if (nst < 2) {
-    set_error("tvl_gemv_q8: not enough shared memory");
-    return TVL_E_UNSUPPORTED;
-  }
-  a.nst = nst;
-  a.sm_ring = 0;
-  a.sm_bars = nst * kStageBytes;
-  a.sm_x = a.sm_bars + bars;
-  a.sm_seg = a.sm_x + xbytes;
-  a.sm_misc = a.sm_seg + segb;
-  const int smem = a.sm_misc + misc;
-  TVL_CK(cudaFuncSetAttribute((const void*)gemv_stream_kernel<true>,
-                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-  gemv_stream_kernel<true><<<G, kThreads, smem, s>>>(a);
-  TVL_CK(cudaGetLastError());
-  return TVL_OK;
+  return launch_stream<true, false>(a, di, (cudaStream_t)stream, "tvl_gemv_q8");
 }
 
 // ---- weight-only 4-bit rows: quantization and GEMV ---------------------------------
@@ -556,11 +620,9 @@ extern "C" tvl_status tvl_gemv_q4(const void* Wq4, const float* x, float* y, int
     set_error("tvl_gemv_q4: a packed row must fit one 16 KB stage (d_in <= 32736)");
     return TVL_E_UNSUPPORTED;
   }
-  cudaStream_t s = (cudaStream_t)stream;
-  int dev = 0, sms = 0, max_optin = 0;
-  TVL_CK(cudaGetDevice(&dev));
-  TVL_CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-  TVL_CK(cudaDeviceGetAttribute(&max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev));
+  DevInfo di;
+  tvl_status st = dev_info("tvl_gemv_q4", &di);
+  if (st != TVL_OK) return st;
   GemvArgs a{};
   a.W = reinterpret_cast<const float*>(Wq4);
   a.x = x;
@@ -570,26 +632,5 @@ extern "C" tvl_status tvl_gemv_q4(const void* Wq4, const float* x, float* y, int
   a.S = 1;
   a.Kc = Kw;
   a.nv = d_out;
-  const int G = d_out < sms ? d_out : sms;
-  const int xbytes = (int)a128(4LL * d_in), segb = (int)a128(kMaxSegParts * 4);
-  const int bars = (int)a128(kRingBarBytes);
-  const int misc = 128;
-  int nst = (max_optin - xbytes - segb - bars - misc) / kStageBytes;
-  if (nst > kMaxStages) nst = kMaxStages;
-  if (nst < 2) {
-    set_error("tvl_gemv_q4: not enough shared memory");
-    return TVL_E_UNSUPPORTED;
-  }
-  a.nst = nst;
-  a.sm_ring = 0;
-  a.sm_bars = nst * kStageBytes;
-  a.sm_x = a.sm_bars + bars;
-  a.sm_seg = a.sm_x + xbytes;
-  a.sm_misc = a.sm_seg + segb;
-  const int smem = a.sm_misc + misc;
-  TVL_CK(cudaFuncSetAttribute((const void*)gemv_stream_kernel<false, true>,
-                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-  gemv_stream_kernel<false, true><<<G, kThreads, smem, s>>>(a);
-  TVL_CK(cudaGetLastError());
-  return TVL_OK;
+  return launch_stream<false, true>(a, di, (cudaStream_t)stream, "tvl_gemv_q4");
 }

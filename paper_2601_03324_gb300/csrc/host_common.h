@@ -29,6 +29,15 @@ struct BlobLayout {
   int64_t g_att = 0, wq = 0, wk = 0, wv = 0, wo = 0, g_ffn = 0, w1 = 0, w3 = 0, w2 = 0;  // in a layer
 };
 
+// Every device and pinned-host allocation of the library goes through these:
+// they count the allocations held (tvl_debug_live_allocations) and can be told
+// to fail one attempt (tvl_debug_fail_allocation), so that tests can reach
+// every failure point of the allocating calls and check their clean-up.
+cudaError_t lib_malloc(void** p, size_t bytes);
+void lib_free(void* p);
+cudaError_t lib_host_alloc(void** p, size_t bytes, unsigned flags);
+void lib_free_host(void* p);
+
 bool config_valid(const tvl_config* c);
 BlobLayout blob_layout(const tvl_config* c, bool tied);
 

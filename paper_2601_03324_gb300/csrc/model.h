@@ -28,7 +28,12 @@ struct tvl_model {
   int vs = 0;
   int smem_bytes = 0;
   int* err_host = nullptr;  // pinned, mapped: the kernel writes its error code here too
-  unsigned epoch = 1;       // tag of the next launch's first exchange (0 = never written)
+  // Tag of the next launch's first exchange. Tags are 32-bit and 0 means never
+  // written; before a launch whose tags would pass 2^32 - 1 the exchange words
+  // [xchg_off, xchg_off + xchg_bytes) of the arena are zeroed and tags start at 1
+  // again, so a tag is never reused while a word may still hold it.
+  uint64_t next_tag = 1;
+  size_t xchg_off = 0, xchg_bytes = 0;
   tvl_status sticky = TVL_OK;
   // multi-token prefill (prefill.cu): created on first use
   void* blas = nullptr;  // cublasHandle_t bound to `stream`

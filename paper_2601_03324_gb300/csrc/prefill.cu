@@ -205,7 +205,7 @@ bool on_device(const void* p) {
 
 void prefill_release(tvl_model* m) {
   if (m->blas) cublasDestroy(static_cast<cublasHandle_t>(m->blas));
-  if (m->pf) cudaFree(m->pf);
+  lib_free(m->pf);
   m->blas = nullptr;
   m->pf = nullptr;
   m->pf_bytes = 0;
@@ -241,7 +241,7 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
                fh = (size_t)S * F;
   const size_t need = 4 * (3 * fx + fqkv + fh13 + fh + d) + 4 * (size_t)S + 256;
   if (!m->pf) {
-    TVL_CK(cudaMalloc((void**)&m->pf, need));
+    TVL_CK(lib_malloc((void**)&m->pf, need));
     m->pf_bytes = need;
   }
   if (!m->blas) {

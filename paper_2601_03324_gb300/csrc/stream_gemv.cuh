@@ -155,6 +155,32 @@ __device__ inline bool wait_bounded(uint64_t* bar, uint32_t par, const int* err,
 // CTA's stage plan, false at the end. Before reusing a slot it waits for the
 // consumers to release it; before returning it waits for every copy it queued
 // (a CTA must not exit with copies into its shared memory in flight).
+// A second walk over the same schedule, kPrefetchAhead stages ahead of the
+// copies: each of its stages is prefetched into L2, so that the HBM reads of
+// a stage are done well before its copy into shared memory is issued.
+constexpr int kPrefetchAhead = 12;
+template <class Sched>
+struct PrefetchCursor {
+  Sched sched;
+  const float* W = nullptr;
+  StagePlan p;
+  int j = 0;
+  bool valid = false;
+  __device__ void start() {
+    valid = sched.next(W, p);
+    j = 0;
+  }
+  __device__ void step() {  // prefetch the next stage of the schedule, if any
+    while (valid && j >= p.nstages) {
+      valid = sched.next(W, p);
+      j = 0;
+    }
+    if (!valid) return;
+    const StageDesc s = stage_desc(p, j++);
+    bulk_prefetch_l2(W + (size_t)s.row * p.K + s.c0, (uint32_t)(s.nrows * (s.c1 - s.c0)) * 4u);
+  }
+};
+
 template <class Sched>
 __device__ inline void run_producer(const Ring& r, Sched& sched, int* err, int* err_host,
                                     volatile int* s_abort) {
@@ -163,8 +189,13 @@ __device__ inline void run_producer(const Ring& r, Sched& sched, int* err, int* 
   const float* W = nullptr;
   StagePlan p;
   bool ok = true;
+  PrefetchCursor<Sched> ahead;
+  ahead.sched = sched;
+  ahead.start();
+  for (int i = 0; i < kPrefetchAhead; ++i) ahead.step();
   while (ok && sched.next(W, p)) {
     for (int j = 0; j < p.nstages; ++j, ++g) {
+      ahead.step();
       const int slot = (int)(g % (uint32_t)r.nst);
       if (g >= (uint32_t)r.nst) {
         bool to = false;
@@ -386,15 +417,30 @@ __device__ __forceinline__ float row_partial_q4(const int* c0, const float4* x4,
 // applies the limit): first until the producer has queued that stage into the
 // slot, then until its bytes have landed. Returns the same answer in every
 // lane of the warp.
+__device__ inline bool warp_wait_full_at(const Ring& r, int slot, uint32_t par, uint32_t gs,
+                                         bool need_seq, int* err, int* err_host,
+                                         volatile int* s_abort);
+
 __device__ inline bool warp_wait_full(const Ring& r, int slot, uint32_t gs, int* err,
                                       int* err_host, volatile int* s_abort) {
+  return warp_wait_full_at(r, slot, (gs / (uint32_t)r.nst) & 1u, gs, true, err, err_host,
+                           s_abort);
+}
+
+// The same wait with the slot's parity given (gs / nst, odd or even).
+// need_seq: the stage that used the slot before (gs - nst) may still be on its
+// way (it belongs to the same phase), so the barrier may be a whole lap behind
+// and its parity alone cannot tell the laps apart; the sequence word can.
+__device__ inline bool warp_wait_full_at(const Ring& r, int slot, uint32_t par, uint32_t gs,
+                                         bool need_seq, int* err, int* err_host,
+                                         volatile int* s_abort) {
   uint64_t* bar = &r.full[slot];
-  const uint32_t par = (gs / (uint32_t)r.nst) & 1u;
   // usual case: the stage was queued long ago and has landed
-  if (__all_sync(0xffffffffu, r.seq[slot] == (int)(gs + 1u) && mbar_test_wait(bar, par)))
+  if (__all_sync(0xffffffffu, (!need_seq || r.seq[slot] == (int)(gs + 1u)) &&
+                                  mbar_test_wait(bar, par)))
     return true;
   bool ok = true;
-  if (r.seq[slot] != (int)(gs + 1u)) {
+  if (need_seq && r.seq[slot] != (int)(gs + 1u)) {
     const bool leader = (threadIdx.x & 31) == 0;
     const uint64_t t0 = leader ? globaltimer_ns() : 0;
     for (uint32_t it = 1; r.seq[slot] != (int)(gs + 1u); ++it) {
@@ -608,7 +654,7 @@ __device__ __forceinline__ float warp_sum_transposed(float (&v)[N], int lane) {
 // row r + 1 with vector b when r + 1 < R.
 template <int R, int kB, class Put>
 __device__ __forceinline__ void rows_times_vectors(const float* w, int ncols, const float* x,
-                                                   int vs, int lane, Put put) {
+                                                   int vs, int lane, bool pairs, Put put) {
   const int n4 = ncols >> 2, vs4 = vs >> 2;
   const float4* w4 = reinterpret_cast<const float4*>(w);
   const float4* x4 = reinterpret_cast<const float4*>(x);
@@ -650,10 +696,26 @@ __device__ __forceinline__ void rows_times_vectors(const float* w, int ncols, co
     v[i] = i >= R * kB ? 0.f : kWide ? (acc[i][0] + acc[i][A > 1 ? 1 : 0]) + (acc[i][A > 2 ? 2 : 0] + acc[i][A > 3 ? 3 : 0]) : acc[i][0];
   const float t = warp_sum_transposed<N>(v, lane);
   // the next row's sum for the same vector, for paired rows
-  const float tn = __shfl_down_sync(0xffffffffu, t, kB * (32 / N));
+  const float tn = pairs ? __shfl_down_sync(0xffffffffu, t, kB * (32 / N)) : 0.f;
   const int idx = lane / (32 / N);
   if (lane % (32 / N) == 0 && idx < R * kB) put(idx / kB, idx % kB, t, tn);
 }
+
+// The consumers' position in the stage stream, kept without divisions: g
+// stages consumed so far, slot = g mod nst, lap = g / nst, w7 = g mod 7.
+struct StageCursor {
+  uint32_t g = 0, lap = 0;
+  int slot = 0, w7 = 0;
+  __device__ __forceinline__ void advance(int n, int nst) {
+    g += (uint32_t)n;
+    slot += n;
+    while (slot >= nst) {
+      slot -= nst;
+      ++lap;
+    }
+    w7 = (w7 + n) % kConsumerWarps;
+  }
+};
 
 // consume_phase for kB input vectors at once (vector b at xs + b * vs): the
 // same stages, each weight read once from the ring for all kB products.
@@ -661,16 +723,23 @@ __device__ __forceinline__ void rows_times_vectors(const float* w, int ncols, co
 // epi.store_pair_b(row, b, value, value of row + 1) paired rows. Deferred rows
 // leave kB partials per segment in seg, added in segment order.
 template <int kB, class Epi>
-__device__ inline bool consume_phase_b(const Ring& r, uint32_t& g, const StagePlan& p,
+__device__ inline bool consume_phase_b(const Ring& r, StageCursor& cur, const StagePlan& p,
                                        const float* xs, int vs, float* seg, Epi& epi, int* err,
                                        int* err_host, volatile int* s_abort) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   bool ok = true;
-  int j = (int)((warp + kConsumerWarps - (int)(g % kConsumerWarps)) % kConsumerWarps);
+  const bool pairs = p.gran == 2;
+  int j = warp - cur.w7;
+  if (j < 0) j += kConsumerWarps;
+  int slot = cur.slot + j;
+  uint32_t lap = cur.lap;
+  while (slot >= r.nst) {
+    slot -= r.nst;
+    ++lap;
+  }
   for (; j < p.nstages && ok; j += kConsumerWarps) {
-    const uint32_t gs = g + (uint32_t)j;
-    const int slot = (int)(gs % (uint32_t)r.nst);
-    if (!warp_wait_full(r, slot, gs, err, err_host, s_abort)) {
+    const uint32_t gs = cur.g + (uint32_t)j;
+    if (!warp_wait_full_at(r, slot, lap & 1u, gs, j >= r.nst, err, err_host, s_abort)) {
       ok = false;
       break;
     }
@@ -678,7 +747,7 @@ __device__ inline bool consume_phase_b(const Ring& r, uint32_t& g, const StagePl
     const int ncols = s.c1 - s.c0;
     const float* st = reinterpret_cast<const float*>(r.buf + (size_t)slot * kStageBytes);
     const float* xb = xs + s.c0;
-    const int part = j % p.spr;
+    const int part = p.spr == 1 ? 0 : j % p.spr;
     int ri = 0;
     auto put_at = [&](int r0) {
       return [&, r0](int rr, int b, float v, float vn) {
@@ -692,18 +761,23 @@ __device__ inline bool consume_phase_b(const Ring& r, uint32_t& g, const StagePl
       };
     };
     for (; ri + 4 <= s.nrows; ri += 4)
-      rows_times_vectors<4, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, put_at(ri));
+      rows_times_vectors<4, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, pairs, put_at(ri));
     if (s.nrows - ri == 3) {
-      rows_times_vectors<3, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, put_at(ri));
+      rows_times_vectors<3, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, pairs, put_at(ri));
     } else if (s.nrows - ri == 2) {
-      rows_times_vectors<2, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, put_at(ri));
+      rows_times_vectors<2, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, pairs, put_at(ri));
     } else if (s.nrows - ri == 1) {
-      rows_times_vectors<1, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, put_at(ri));
+      rows_times_vectors<1, kB>(st + (size_t)ri * ncols, ncols, xb, vs, lane, pairs, put_at(ri));
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(&r.empty[slot]);  // stage free for the producer
+    slot += kConsumerWarps;
+    while (slot >= r.nst) {
+      slot -= r.nst;
+      ++lap;
+    }
   }
-  g += (uint32_t)p.nstages;
+  cur.advance(p.nstages, r.nst);
   if (named_bar_or(kBarConsumers, kConsumerThreads, !ok)) {
     if (tid == 0) *s_abort = 1;
     return false;

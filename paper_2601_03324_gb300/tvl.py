@@ -42,8 +42,8 @@ class ModelInfo(ctypes.Structure):
         ("streamed_bytes", ctypes.c_int64), ("grid", ctypes.c_int32),
         ("threads", ctypes.c_int32), ("smem_bytes", ctypes.c_int32),
         ("ring_stages", ctypes.c_int32), ("stage_bytes", ctypes.c_int32),
-        ("tied", ctypes.c_int32), ("barriers_per_step", ctypes.c_int32),
-        ("max_batch", ctypes.c_int32),
+        ("tied", ctypes.c_int32), ("exchanges_per_step", ctypes.c_int32),
+        ("max_batch", ctypes.c_int32), ("next_tag", ctypes.c_int64),
     ]
 
 
@@ -86,6 +86,10 @@ def _load():
     L.tvl_gemv_q4.argtypes = [P, P, P, i32, i32, P]
     L.tvl_gemv_noalloc.restype = st
     L.tvl_gemv_noalloc.argtypes = [P, P, P, i32, i32, P]
+    L.tvl_gemv_status.restype = st
+    L.tvl_gemv_status.argtypes = [P]
+    L.tvl_selftest_gemv_timeout.restype = st
+    L.tvl_selftest_gemv_timeout.argtypes = [P, P, P, i32, i32, P]
     L.tvl_sync.restype = st
     L.tvl_sync.argtypes = [P]
     L.tvl_free.restype = None
@@ -100,6 +104,12 @@ def _load():
     L.tvl_step_times.argtypes = [P, P, i32]
     L.tvl_selftest_barrier_timeout.restype = st
     L.tvl_selftest_barrier_timeout.argtypes = [i32]
+    L.tvl_debug_fail_allocation.restype = None
+    L.tvl_debug_fail_allocation.argtypes = [i32]
+    L.tvl_debug_live_allocations.restype = i64
+    L.tvl_debug_live_allocations.argtypes = []
+    L.tvl_debug_set_next_tag.restype = st
+    L.tvl_debug_set_next_tag.argtypes = [P, ctypes.c_uint64]
     return L
 
 
@@ -107,10 +117,12 @@ lib = _load()
 
 EXPORTED = ["tvl_blob_bytes", "tvl_load", "tvl_load_file", "tvl_forward", "tvl_decode_greedy",
             "tvl_forward_batch", "tvl_decode_greedy_batch", "tvl_prefill",
-            "tvl_gemv", "tvl_gemv_noalloc", "tvl_q8_bytes", "tvl_quantize_q8", "tvl_gemv_q8",
+            "tvl_gemv", "tvl_gemv_noalloc", "tvl_gemv_status", "tvl_selftest_gemv_timeout",
+            "tvl_q8_bytes", "tvl_quantize_q8", "tvl_gemv_q8",
             "tvl_q4_bytes", "tvl_quantize_q4", "tvl_gemv_q4",
             "tvl_sync", "tvl_free", "tvl_status_string", "tvl_last_error",
-            "tvl_get_info", "tvl_step_times", "tvl_selftest_barrier_timeout"]
+            "tvl_get_info", "tvl_step_times", "tvl_selftest_barrier_timeout",
+            "tvl_debug_fail_allocation", "tvl_debug_live_allocations", "tvl_debug_set_next_tag"]
 
 
 def status_string(s: int) -> str:
@@ -160,6 +172,19 @@ def tvl_gemv_noalloc(W, x, y, d_out: int, d_in: int, stream: int = 0):
     _check(lib.tvl_gemv_noalloc(ctypes.c_void_p(_addr(W)), ctypes.c_void_p(_addr(x)),
                                 ctypes.c_void_p(_addr(y)), int(d_out), int(d_in),
                                 ctypes.c_void_p(int(stream))), "tvl_gemv_noalloc")
+
+
+def tvl_gemv_status(stream: int = 0) -> int:
+    """Waits for `stream`; the standalone GEMV kernels' error since the last
+    query (TVL_E_TIMEOUT) or OK. Returns the status, does not raise."""
+    return lib.tvl_gemv_status(ctypes.c_void_p(stream))
+
+
+def tvl_selftest_gemv_timeout(W, x, y, d_out: int, d_in: int, stream: int = 0) -> int:
+    """Returns the status the self-test reports (TVL_E_TIMEOUT expected)."""
+    return lib.tvl_selftest_gemv_timeout(ctypes.c_void_p(_addr(W)), ctypes.c_void_p(_addr(x)),
+                                         ctypes.c_void_p(_addr(y)), int(d_out), int(d_in),
+                                         ctypes.c_void_p(stream))
 
 
 def tvl_q8_bytes(rows: int, cols: int) -> int:

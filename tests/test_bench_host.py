@@ -61,7 +61,7 @@ def test_single_rank_needs_no_process_group():
 
 def _ref_args(**kw):
     a = dict(gpus=2, steps=1, warmup=0, impl="reference", workload="tiny", no_e2e=False,
-             no_cpu_baseline=False, cpu_seconds=1.0, gemv_sweep=False)
+             no_cpu_baseline=False, cpu_seconds=1.0, gemv_sweep=False, weights="f32", batch=1)
     a.update(kw)
     return argparse.Namespace(**a)
 
@@ -84,3 +84,40 @@ def test_reference_arm_rank0_line(capsys):
     assert line["value"] > 0 and line["unit"] == "tokens/s" and line["higher_is_better"]
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 1
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
+
+
+def test_timed_windows_keep_the_sequence_mean_position():
+    import bench
+    # 20 steps of a 256-step sequence: positions 118..137, mean 127.5
+    assert bench.timed_windows(256, 20, 0) == [(118, 20)]
+    for seq, k, pos0 in ((256, 20, 0), (256, 600, 0), (64, 20, 0), (128, 20, 896), (16, 20, 0),
+                         (256, 256, 0), (256, 1, 0), (256, 255, 0)):
+        wins = bench.timed_windows(seq, k, pos0)
+        assert sum(n for _, n in wins) == k
+        steps = [p + i for (p, n) in wins for i in range(n)]
+        assert all(pos0 <= q < pos0 + seq for q in steps)
+        # every window is consecutive positions inside one sequence, and the
+        # timed steps' mean position is the sequence's (up to half a step)
+        assert abs(sum(steps) / k - (pos0 + (seq - 1) / 2)) <= 0.5
+
+
+def test_window_start_tokens_come_from_the_fill_run():
+    import numpy as np
+    import bench
+    fill = np.arange(1000, 1256)  # fill[s] = the greedy token after step s
+    wins = [(0, 256), (118, 20)]
+    assert bench.window_starts(wins, 0, [1], fill) == [[1], [1117]]
+    fillb = np.stack([fill, fill + 5000], axis=1)  # two sequences
+    assert bench.window_starts([(118, 20)], 0, [1, 100], fillb) == [[1117, 6117]]
+    assert bench.positions_of([(0, 256), (0, 256), (118, 20)]) == [[0, 255], [118, 137]]
+
+
+def test_reference_arm_config_equals_the_gpu_arms(capsys):
+    import bench
+    from paper_2601_03324_gb300 import synth
+    cfg = synth.model_config("tiny")
+    assert bench.run_reference(_ref_args(steps=3, gpus=1), cfg, rank=0, world=1) == 0
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    wins = bench.timed_windows(64, 3, 0)
+    assert line["config"] == bench.workload_config("tiny", cfg, 1, "f32", bench.positions_of(wins))
+    assert line["config"]["positions"] == [[30, 32]]

@@ -25,6 +25,10 @@ def tvl():
 
 @pytest.mark.parametrize("shape", SHAPES, ids=lambda s: f"{s[0]}x{s[1]}")
 def test_noalloc_matches_tvl_gemv_on_two_consecutive_calls(tvl, shape):
+    """Same kernel, same split, partials summed in the same order: the output
+    equals tvl_gemv's bit for bit, on two calls in a row (the second finds the
+    counters the first left), and lies within the GEMV bound of the oracle."""
+    import oracle
     M, K = shape
     W, x = synth.gemv_operands(M, K, 11)
     dW, dx = torch.from_numpy(W).cuda(), torch.from_numpy(x).cuda()
@@ -33,16 +37,36 @@ def test_noalloc_matches_tvl_gemv_on_two_consecutive_calls(tvl, shape):
     tvl.tvl_gemv(dW.data_ptr(), dx.data_ptr(), ref.data_ptr(), M, K, s.cuda_stream)
     s.synchronize()
     y_ref = ref.cpu().numpy()
+    truth = oracle.gemv(W, x)
     bound = gemv_bound(W, x)
-    outs = []
-    for _ in range(2):  # the counters must be back at zero for the second call
+    for _ in range(2):
         y = torch.full((M,), float("nan"), device="cuda")
         tvl.tvl_gemv_noalloc(dW.data_ptr(), dx.data_ptr(), y.data_ptr(), M, K, s.cuda_stream)
         s.synchronize()
-        outs.append(y.cpu().numpy())
-    for y in outs:
-        assert np.all(np.isfinite(y))
-        assert np.all(np.abs(y - y_ref) <= bound), float(np.abs(y - y_ref).max())
+        got = y.cpu().numpy()
+        assert np.array_equal(got, y_ref)
+        assert np.all(np.abs(got - truth) <= bound), float(np.abs(got - truth).max())
+    assert tvl.tvl_gemv_status(s.cuda_stream) == tvl.OK
+
+
+def test_noalloc_allocates_no_device_memory(tvl):
+    """After the first call on the device (the one-time setup), further calls
+    leave the device's free memory and the library's allocation count as they
+    were."""
+    M, K = 768, 768  # split along K: the static scratch is in use
+    W, x = synth.gemv_operands(M, K, 12)
+    dW, dx = torch.from_numpy(W).cuda(), torch.from_numpy(x).cuda()
+    y = torch.empty(M, device="cuda")
+    s = torch.cuda.Stream()
+    tvl.tvl_gemv_noalloc(dW.data_ptr(), dx.data_ptr(), y.data_ptr(), M, K, s.cuda_stream)
+    s.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    live0 = tvl.lib.tvl_debug_live_allocations()
+    for _ in range(5):
+        tvl.tvl_gemv_noalloc(dW.data_ptr(), dx.data_ptr(), y.data_ptr(), M, K, s.cuda_stream)
+    s.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    assert tvl.lib.tvl_debug_live_allocations() == live0
 
 
 def test_noalloc_rejects_bad_arguments(tvl):
