@@ -378,9 +378,14 @@ def gemv_sweep(args):
     import torch
     from paper_2601_03324_gb300 import synth, tvl
     torch.cuda.set_device(0)
-    l2 = torch.cuda.get_device_properties(0).L2_cache_size
+    props = torch.cuda.get_device_properties(0)
+    l2 = props.L2_cache_size
     s = torch.cuda.Stream()
     out = []
+    uuid = getattr(props, "uuid", None)
+    uuid = f"GPU-{uuid}" if uuid and not str(uuid).startswith("GPU-") else (str(uuid) if uuid else None)
+    clocks = Clocks(0, uuid)
+    t_wall0 = time.time()
     for i, (M, K) in enumerate(synth.GEMV_SHAPES):
         W, x = synth.gemv_operands(M, K, i)
         packed = {"q8": (tvl.tvl_q8_bytes, tvl.tvl_quantize_q8, tvl.tvl_gemv_q8),
@@ -421,6 +426,7 @@ def gemv_sweep(args):
         out.append({"shape": [M, K], "us": us, "GB/s": nbytes / us / 1e3,
                     "copies": copies, "fits_l2": wbytes <= l2})
         del dW, g
+    clk = clocks.stop(t_wall0, time.time())
     peak, src = measured_peaks()
     for o in out:
         o["frac_of_" + src + "_hbm"] = o["GB/s"] / peak
@@ -428,7 +434,11 @@ def gemv_sweep(args):
             "not an HBM one)" if args.hot else
             "cold: W rotated over copies totalling 3x L2, so every call reads it from HBM")
     print(json.dumps({"gemv_sweep": out, "weights": args.weights, "mode": mode,
-                      "peak_gbs": peak, "peak_source": src}), flush=True)
+                      "peak_gbs": peak, "peak_source": src, "reps_per_shape": 200,
+                      "timing": "200 calls captured in one CUDA graph, CUDA events around "
+                                "one replay, divided by 200",
+                      "clocks": dict(clk, window="the whole sweep, set-up included")}),
+          flush=True)
 
 
 def main():

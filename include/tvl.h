@@ -161,8 +161,11 @@ tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n, int32_t s
  * (TMA bulk staging) needs W and x 16-byte aligned and d_in % 4 == 0 and
  * d_in <= 16384; other shapes take a plain per-row kernel. Deterministic: the
  * same inputs give the same bits. A per-stream scratch buffer (a few KB) is
- * allocated on first use for short-and-wide shapes and kept until exit;
- * concurrent calls on different streams are safe. */
+ * allocated on first use for matrices with fewer rows than the GPU has SMs
+ * (split along d_in) and kept until exit; concurrent calls on different
+ * streams are safe. The kernel is launched with a programmatic dependency on
+ * the stream's previous kernel: it may start while that kernel finishes, and
+ * reads x, writes y and copies W only once that kernel has completed. */
 tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t d_out, int32_t d_in,
                     void* stream);
 
@@ -227,7 +230,7 @@ tvl_status tvl_gemv_q4(const void* Wq4, const float* x, float* y, int32_t d_out,
  * split, bit-identical output). The split-K scratch is one static module
  * array of 48 KB per device (8192 partials, 4096 row counters), not
  * allocated memory. A shape whose split needs more (never on a 152-SM GB300:
- * at most 4864 partials and 2431 rows) returns TVL_E_UNSUPPORTED with the
+ * at most 302 partials and 151 rows) returns TVL_E_UNSUPPORTED with the
  * sizes in tvl_last_error(); use tvl_gemv for it.
  * The FIRST call on a device does a one-time setup: it looks up the array's
  * device address, zeroes its counters on `stream` and waits for that, so make

@@ -33,9 +33,40 @@ __global__ void wait_selftest_kernel(unsigned long long* word, int* err,
   vote_ok(ok, &s_abort);
 }
 
+// W[r][j] *= g[j] for rows [0, rows) of W [rows x cols] (cols % 4 == 0): an
+// RMSNorm gain folded into the columns of a matrix that reads the normalised
+// vector, W ((x * g) r) = r (W diag(g)) x.
+__global__ void scale_columns_kernel(float* __restrict__ W, long long rows, int cols,
+                                     const float* __restrict__ g) {
+  const int c4 = cols >> 2;
+  const long long n = rows * c4;
+  float4* w4 = reinterpret_cast<float4*>(W);
+  const float4* g4 = reinterpret_cast<const float4*>(g);
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n;
+       i += (long long)gridDim.x * blockDim.x) {
+    const float4 gv = g4[i % c4];
+    float4 v = w4[i];
+    v.x *= gv.x;
+    v.y *= gv.y;
+    v.z *= gv.z;
+    v.w *= gv.w;
+    w4[i] = v;
+  }
+}
+
 }  // namespace tvl
 
 namespace {
+
+tvl_status scale_columns(unsigned char* W, long long rows, int cols, const unsigned char* g,
+                         cudaStream_t st) {
+  const long long n = rows * (cols / 4);
+  const int blocks = (int)std::min<long long>((n + 255) / 256, 4096);
+  scale_columns_kernel<<<blocks, 256, 0, st>>>(reinterpret_cast<float*>(W), rows, cols,
+                                               reinterpret_cast<const float*>(g));
+  TVL_CK(cudaGetLastError());
+  return TVL_OK;
+}
 
 struct SmemPlan {
   int ring, bars, xs, vec, seg, att, misc, total, nst;
@@ -399,6 +430,22 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
     lib_free(tmp);
     if (st != TVL_OK) return fail(st);
   }
+  if (!q8) {
+    // float32 rows: the RMSNorm gains go into the columns of the matrices that
+    // read the normalised vectors ([Wq|Wk|Wv] g_att, W1/W3 g_ffn, and the
+    // classifier g_final unless it is the embedding table), so that the
+    // kernel's phase input is x itself. (8-bit rows keep the gains apart: their
+    // codes are those of the matrices as given.)
+    for (int l = 0; l < L && st == TVL_OK; ++l) {
+      unsigned char* lw = m->arena + o_w + bl.l0 + (size_t)l * bl.stride;
+      st = scale_columns(lw + bl.wq, d + 2LL * kvd, d, lw + bl.g_att, m->stream);
+      if (st == TVL_OK) st = scale_columns(lw + bl.w1, 2LL * F, d, lw + bl.g_ffn, m->stream);
+    }
+    if (st == TVL_OK && !tied)
+      st = scale_columns(m->arena + o_w + bl.Wcls, V, d, m->arena + o_w + bl.g_final, m->stream);
+    if (st == TVL_OK) st = ck(cudaStreamSynchronize(m->stream), "cudaStreamSynchronize(gains)");
+    if (st != TVL_OK) return fail(st);
+  }
 
   // ---- RoPE table: pair i at position p turns by p * theta^(-2i/hd) ------------------
   {
@@ -462,6 +509,8 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   a.att_stride = att_stride;
   a.nch_cap = nch_cap;
   a.eps = (float)cfg->norm_eps;
+  a.gains_folded = !q8;
+  a.final_gain_folded = !q8 && !tied;
   a.att_scale = (float)(1.0 / std::sqrt((double)hd));
   a.kv_seq = (long long)kv_seq;
   a.wait_limit_ns = kWaitLimitNs;

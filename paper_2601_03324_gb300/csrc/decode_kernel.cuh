@@ -78,6 +78,11 @@ struct DecodeArgs {
   int d, F, V, L, H, Hkv, hd, kvd, S, G;
   int att_stride, nch_cap;
   float eps, att_scale;
+  // RMSNorm gains already multiplied into the columns of the matrices that
+  // read the normalised vector (the layers' [Wq|Wk|Wv] and W1/W3; the
+  // classifier when it is not the embedding table): the phase input is then x
+  // itself, and no gain is loaded on the way from an exchange to a GEMV
+  bool gains_folded, final_gain_folded;
   // this launch
   int start_pos, n_steps, final_token;
   // B sequences decode in lockstep at the same positions: sequence b's words
@@ -230,8 +235,8 @@ __device__ inline bool poll_pairs_at(int npairs, Addr addr, unsigned tag, const 
 
 // Poll quads j = tid, tid + 224, ... (nquads quads of four consecutive words),
 // Q quads (2 Q 16-byte loads) in flight per thread, and load quad j mod n4 of
-// aux (the RMSNorm gains) for each while the polls are out; fn(j, v, aux quad)
-// takes each ready quad. Returns false if this thread gave up.
+// aux (the RMSNorm gains; null: all ones) for each while the polls are out;
+// fn(j, v, aux quad) takes each ready quad. Returns false if this thread gave up.
 template <int Q, class Fn>
 __device__ inline bool poll_quads(const unsigned long long* src, int nquads, unsigned tag,
                                   const float4* aux, int n4, const Poll& c, Fn fn) {
@@ -251,7 +256,7 @@ __device__ inline bool poll_quads(const unsigned long long* src, int nquads, uns
 #pragma unroll
     for (int b = 0; b < Q; ++b) {
       const int j = base + b * kConsumerThreads;
-      if (j < nquads) ax[b] = __ldg(aux + j % n4);
+      if (j < nquads) ax[b] = aux ? __ldg(aux + j % n4) : make_float4(1.f, 1.f, 1.f, 1.f);
     }
     PollClock clk;
     while (true) {
@@ -753,6 +758,8 @@ struct DecodeSched {
   const StagePlan* plans;
   uint32_t refill_delay_ns = kRefillDelayNs;
   int s = 0, l = 0, k = 0;
+  int prefetch_ahead = kPrefetchAhead;  // stages prefetched into L2 ahead of the copies
+  __device__ void before_copies() {}  // launched without a programmatic dependency
   __device__ bool next(const float*& W, StagePlan& p) {
     if (s >= a->n_steps) return false;
     if (l < a->L) {
@@ -838,7 +845,8 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
   auto norm_local = [&](const float* gain, float(&ss)[kB]) {
     const float4* g4 = reinterpret_cast<const float4*>(gain);
     for (int j = tid; j < kB * n4; j += kConsumerThreads)
-      norm_quad(j, reinterpret_cast<const float4*>(xs)[j], __ldg(g4 + j % n4), ss);
+      norm_quad(j, reinterpret_cast<const float4*>(xs)[j],
+                g4 ? __ldg(g4 + j % n4) : make_float4(1.f, 1.f, 1.f, 1.f), ss);
   };
   // r_b from every thread's share of ss_b: warp sums go to red, and the block
   // vote that follows the exchange publishes them (and x, vec)
@@ -915,7 +923,9 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
         if (k == 0 || k == 2) {
           // x += (the previous phase's published output); the input is x * g,
           // scaled by r in the epilogue
-          const float* gain = reinterpret_cast<const float*>(lw + (k == 0 ? a.o_gatt : a.o_gffn));
+          const float* gain =
+              a.gains_folded ? nullptr
+                             : reinterpret_cast<const float*>(lw + (k == 0 ? a.o_gatt : a.o_gffn));
           float ss[kB];
 #pragma unroll
           for (int b = 0; b < kB; ++b) ss[b] = 0.f;
@@ -971,8 +981,9 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
 #pragma unroll
       for (int b = 0; b < kB; ++b) ss[b] = 0.f;
       bool ok = true;
-      if (a.L > 0) ok = add_published(a.x_f, es + per_step - 2, a.g_final, ss);
-      else norm_local(a.g_final, ss);
+      const float* gf = a.final_gain_folded ? nullptr : a.g_final;
+      if (a.L > 0) ok = add_published(a.x_f, es + per_step - 2, gf, ss);
+      else norm_local(gf, ss);
       if (!norm_scales(ok, ss, rs)) return false;
     }
     EpiArgmax<kB> ea{a.logits, a.V, {rs[0], rs[1], rs[2], rs[3]}};

@@ -25,6 +25,11 @@ using namespace tvl;
 
 namespace tvl {
 
+// The standalone GEMV copies its stages without L2 prefetches ahead of them:
+// measured over the sweep shapes, prefetching 4 or 12 stages ahead was slower
+// on every shape (the copies already keep up to 12 stages in flight per SM).
+constexpr int kGemvPrefetchAhead = 0;
+
 struct GemvArgs {
   const float* W;
   const float* x;
@@ -49,12 +54,25 @@ struct EpiPart {
   }
 };
 
-// The single phase of a standalone GEMV.
+// The single phase of a standalone GEMV. Launched with a programmatic
+// dependency on the stream's previous kernel: its first copies wait for that
+// kernel (the L2 prefetches before them do not).
 struct GemvSched {
   const float* W;
   uint32_t refill_delay_ns;
   StagePlan p;
   bool given;
+  int prefetch_ahead;  // stages prefetched into L2 ahead of the copies
+  // x [K] goes into shared memory by one bulk copy ahead of the weights
+  float* xs;
+  const float* x;
+  uint32_t xbytes;
+  uint64_t* xbar;
+  __device__ void before_copies() {
+    grid_wait_dependencies();
+    mbar_arrive_expect_tx(xbar, xbytes);
+    bulk_g2s(xs, x, xbytes, xbar, l2_evict_last());
+  }
   __device__ bool next(const float*& w, StagePlan& plan) {
     if (given) return false;
     given = true;
@@ -74,6 +92,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   r.seq = reinterpret_cast<volatile int*>(r.empty + a.nst);
   r.nst = a.nst;
   volatile int* s_abort = reinterpret_cast<volatile int*>(smem + a.sm_misc);
+  uint64_t* xbar = reinterpret_cast<uint64_t*>(smem + a.sm_misc + 64);
+  float* xs = reinterpret_cast<float*>(smem + a.sm_x);
   const StagePlan p = plan_stages(a.nv, a.Kc, gridDim.x, blockIdx.x);
   if (threadIdx.x == 0) {
     for (int i = 0; i < a.nst; ++i) {
@@ -81,25 +101,29 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
       mbar_init(&r.empty[i], 1);
       r.seq[i] = 0;
     }
+    mbar_init(xbar, 1);
     *s_abort = 0;
     fence_mbar_init();
   }
   __syncthreads();
+  // the stream's next kernel may launch now: with the ring sized to the work
+  // its CTAs can start (and prefetch their rows) beside this one's
+  grid_launch_dependents();
   uint32_t g = 0;
   if (threadIdx.x >= kConsumerThreads) {
     if (threadIdx.x == kConsumerThreads) {
-      GemvSched sched{a.W, 0u, p, false};
+      GemvSched sched{a.W, 0u, p, false, kGemvPrefetchAhead, xs, a.x, 4u * (uint32_t)a.K, xbar};
       if (a.drop_last && blockIdx.x == 0 && sched.p.nstages > 0) --sched.p.nstages;
       run_producer(r, sched, a.err, nullptr, s_abort);
+      // the copy of x has landed before the CTA may exit
+      wait_bounded(xbar, 0, nullptr, nullptr, false, nullptr);
     }
     return;
   }
-  float* xs = reinterpret_cast<float*>(smem + a.sm_x);
   float* seg = reinterpret_cast<float*>(smem + a.sm_seg);
-  const float4* x4 = reinterpret_cast<const float4*>(a.x);
-  for (int j = threadIdx.x; j < (a.K >> 2); j += kConsumerThreads)
-    reinterpret_cast<float4*>(xs)[j] = __ldg(x4 + j);
-  named_bar_sync(kBarConsumers, kConsumerThreads);
+  grid_wait_dependencies();  // y and the scratch may still be in use by the previous kernel
+  const bool xok = consumer_wait_full(xbar, 0, a.err, nullptr, s_abort);
+  if (named_bar_or(kBarConsumers, kConsumerThreads, !xok)) return;
   if (a.S == 1) {
     EpiStore e{a.y};
     consume_phase<true, kQ8, kQ4>(r, g, p, xs, 1, a.Kc, seg, e, a.err, nullptr, s_abort);
@@ -275,9 +299,12 @@ unsigned next_call_id(unsigned* next) {
   return id;
 }
 
+// Chunks along K: only when the matrix has fewer rows than there are SMs
+// (each chunk at least 128 floats, the split a power of two dividing K / 4);
+// otherwise every CTA owns whole rows and no partials cross CTAs.
 int split_for(int M, int K, int G) {
   int S = 1;
-  while ((long long)M * S < 16LL * G && K % (8 * S) == 0 && K / (2 * S) >= 128) S *= 2;
+  while ((long long)M * S < G && K % (8 * S) == 0 && K / (2 * S) >= 128) S *= 2;
   return S;
 }
 
@@ -306,15 +333,29 @@ tvl_status launch_rowwise(const float* W, const float* x, float* y, int M, int K
 
 // Shared memory (ring | barriers | x | segment partials | misc, every region a
 // 128-byte multiple) and launch of gemv_stream_kernel<kQ8, kQ4> for a.nv
-// virtual rows of a.Kc words; a.K floats of x.
+// virtual rows of a.Kc words; a.K floats of x. The ring has as many stages as
+// the busiest CTA copies (up to kMaxStages), the partial scratch only when rows
+// are longer than a stage, so that small matrices leave room on each SM for
+// the next kernel's CTAs. The launch carries a programmatic dependency on the
+// stream's previous kernel (the kernel waits for it before its first copy).
 template <bool kQ8, bool kQ4>
 tvl_status launch_stream(GemvArgs& a, const DevInfo& di, cudaStream_t s, const char* who) {
+  static std::mutex mu;
+  static bool attr_set[kMaxDevices] = {};
   const int G = (int)(a.nv < di.sms ? a.nv : di.sms);
-  const int xbytes = (int)a128(4LL * a.K), segb = (int)a128(kMaxSegParts * 4);
+  int need = 1;
+  bool defer = false;
+  for (int c = 0; c < G; ++c) {
+    const StagePlan pl = plan_stages(a.nv, a.Kc, G, c);
+    need = pl.nstages > need ? pl.nstages : need;
+    defer = defer || pl.defer;
+  }
+  const int xbytes = (int)a128(4LL * a.K), segb = defer ? (int)a128(kMaxSegParts * 4) : 128;
   const int bars = (int)a128(kRingBarBytes);
   const int misc = 128;
   int nst = (di.max_optin - xbytes - segb - bars - misc) / kStageBytes;
   if (nst > kMaxStages) nst = kMaxStages;
+  if (nst > need) nst = need < 2 ? 2 : need;
   if (nst < 2) {
     set_error(std::string(who) + ": not enough shared memory");
     return TVL_E_UNSUPPORTED;
@@ -327,10 +368,27 @@ tvl_status launch_stream(GemvArgs& a, const DevInfo& di, cudaStream_t s, const c
   a.sm_seg = a.sm_x + xbytes;
   a.sm_misc = a.sm_seg + segb;
   const int smem = a.sm_misc + misc;
-  TVL_CK(cudaFuncSetAttribute((const void*)gemv_stream_kernel<kQ8, kQ4>,
-                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-  gemv_stream_kernel<kQ8, kQ4><<<G, kThreads, smem, s>>>(a);
-  TVL_CK(cudaGetLastError());
+  int dev = 0;
+  TVL_CK(cudaGetDevice(&dev));
+  {
+    std::lock_guard<std::mutex> lk(mu);
+    if (!attr_set[dev]) {
+      TVL_CK(cudaFuncSetAttribute((const void*)gemv_stream_kernel<kQ8, kQ4>,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, di.max_optin));
+      attr_set[dev] = true;
+    }
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = dim3(G);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = (size_t)smem;
+  cfg.stream = s;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  TVL_CK(cudaLaunchKernelEx(&cfg, gemv_stream_kernel<kQ8, kQ4>, (const GemvArgs)a));
   return TVL_OK;
 }
 
@@ -409,9 +467,9 @@ extern "C" tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t
 namespace {
 
 // Split-K partials (floats) and per-row arrival counters of tvl_gemv_noalloc.
-// split_for keeps M * S below 32 x the SM count and M below 16 x the SM count
-// whenever S > 1, so on a 152-SM part at most 4864 partials and 2431 counters
-// are live; the sizes below leave room for larger parts.
+// split_for splits only matrices with fewer rows than SMs and keeps M * S
+// below twice the SM count, so on a 152-SM part at most 302 partials and 151
+// counters are live; the sizes below leave room for much larger parts.
 constexpr int kNoAllocPart = 8192;
 constexpr int kNoAllocRows = 4096;
 constexpr size_t kNoAllocBytes = 4 * (size_t)kNoAllocPart + 4 * (size_t)kNoAllocRows;  // 48 KB

@@ -37,8 +37,10 @@ __global__ void embed_rows_kernel(const float* __restrict__ E, const int* __rest
 
 // Row i (one block): x_i += add_i when add is given (the residual update),
 // then out_{i - row0} = RMSNorm(x_i, g) = (x_i * g) * 1/sqrt(mean x_i^2 + eps)
-// (§11.2). Rows [row0, row0 + gridDim.x); out may be add (each row is read
-// in full before it is written).
+// (§11.2); g null: the gain is already in the columns of the next matrix
+// (tvl_load folds it there for float32 rows), so out = x_i * r. Rows
+// [row0, row0 + gridDim.x); out may be add (each row is read in full before it
+// is written).
 __global__ void rmsnorm_rows_kernel(float* x, const float* add, const float* __restrict__ g,
                                     float* out, int row0, int d, float eps) {
   __shared__ float red[kRowThreads / 32];
@@ -60,7 +62,7 @@ __global__ void rmsnorm_rows_kernel(float* x, const float* add, const float* __r
   for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += red[w];
   const float r = 1.0f / sqrtf(tot / (float)d + eps);
   float* o = out + (size_t)blockIdx.x * d;
-  for (int j = threadIdx.x; j < d; j += blockDim.x) o[j] = (xr[j] * g[j]) * r;
+  for (int j = threadIdx.x; j < d; j += blockDim.x) o[j] = (g ? xr[j] * g[j] : xr[j]) * r;
 }
 
 // RoPE on q and k of row i (position start + i): pair (2m, 2m+1) of a head
@@ -267,8 +269,8 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
   const float* pending = nullptr;  // residual update not yet added into X
   for (int l = 0; l < L; ++l) {
     const unsigned char* lw = a.layer0 + (size_t)l * a.layer_stride;
-    const float* g_att = reinterpret_cast<const float*>(lw + a.o_gatt);
-    const float* g_ffn = reinterpret_cast<const float*>(lw + a.o_gffn);
+    const float* g_att = a.gains_folded ? nullptr : reinterpret_cast<const float*>(lw + a.o_gatt);
+    const float* g_ffn = a.gains_folded ? nullptr : reinterpret_cast<const float*>(lw + a.o_gffn);
     const float* Wqkv = reinterpret_cast<const float*>(lw + a.o_wqkv);
     const float* Wo = reinterpret_cast<const float*>(lw + a.o_wo);
     const float* W13 = reinterpret_cast<const float*>(lw + a.o_w13);  // interleaved rows
@@ -297,7 +299,8 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
     pending = XB;
   }
   // the last position: x += (last update), x_b = RMSNorm(x, g_final), logits = Wcls x_b
-  rmsnorm_rows_kernel<<<1, kRowThreads, 0, st>>>(X, pending, a.g_final, XN, n - 1, d, a.eps);
+  rmsnorm_rows_kernel<<<1, kRowThreads, 0, st>>>(X, pending, a.final_gain_folded ? nullptr : a.g_final,
+                                                  XN, n - 1, d, a.eps);
   TVL_CK(cudaGetLastError());
   {
     const float one = 1.f, zero = 0.f;

@@ -81,6 +81,24 @@ __device__ __forceinline__ uint64_t l2_evict_first() {
   return p;
 }
 
+// Programmatic dependent launch: let the next kernel of the stream launch now
+// (its CTAs may start while this grid runs) ...
+__device__ __forceinline__ void grid_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+// ... and wait until the grids this one depends on have completed and their
+// memory is visible (returns at once when there are none).
+__device__ __forceinline__ void grid_wait_dependencies() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// L2 policy for data every CTA reads (an input vector): keep it.
+__device__ __forceinline__ uint64_t l2_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
 __device__ __forceinline__ void named_bar_sync(uint32_t id, uint32_t nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }

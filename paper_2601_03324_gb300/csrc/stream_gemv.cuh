@@ -192,10 +192,13 @@ __device__ inline void run_producer(const Ring& r, Sched& sched, int* err, int* 
   PrefetchCursor<Sched> ahead;
   ahead.sched = sched;
   ahead.start();
-  for (int i = 0; i < kPrefetchAhead; ++i) ahead.step();
+  for (int i = 0; i < sched.prefetch_ahead; ++i) ahead.step();
+  // the first copies may need the grids this one depends on to have finished
+  // (the L2 prefetches above only warm the cache)
+  sched.before_copies();
   while (ok && sched.next(W, p)) {
     for (int j = 0; j < p.nstages; ++j, ++g) {
-      ahead.step();
+      if (sched.prefetch_ahead > 0) ahead.step();
       const int slot = (int)(g % (uint32_t)r.nst);
       if (g >= (uint32_t)r.nst) {
         bool to = false;

@@ -89,7 +89,7 @@ struct Shape {
 // tvl_gemv's K split for short-and-wide matrices (same rule as gemv.cu).
 static int split_for(int M, int K, int G) {
   int S = 1;
-  while ((long long)M * S < 16LL * G && K % (8 * S) == 0 && K / (2 * S) >= 128) S *= 2;
+  while ((long long)M * S < G && K % (8 * S) == 0 && K / (2 * S) >= 128) S *= 2;
   return S;
 }
 

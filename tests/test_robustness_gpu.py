@@ -122,7 +122,7 @@ def test_prefill_allocation_failure_leaves_the_model_usable(tvl):
 
 
 def test_gemv_scratch_allocation_failure_returns_nomem_then_recovers(tvl):
-    M, K = 768, 768  # split along K: tvl_gemv needs its per-stream scratch
+    M, K = 64, 8192  # split along K: tvl_gemv needs its per-stream scratch
     W, x = synth.gemv_operands(M, K, 13)
     dW, dx = torch.from_numpy(W).cuda(), torch.from_numpy(x).cuda()
     y = torch.empty(M, device="cuda")
@@ -142,7 +142,7 @@ def test_gemv_scratch_allocation_failure_returns_nomem_then_recovers(tvl):
     assert np.all(np.abs(y.cpu().numpy() - oracle.gemv(W, x)) <= gemv_bound(W, x))
 
 
-@pytest.mark.parametrize("shape", [(768, 768), (2048, 768), (4096, 4096)],
+@pytest.mark.parametrize("shape", [(64, 8192), (100, 2048), (768, 768), (4096, 4096)],
                          ids=lambda s: f"{s[0]}x{s[1]}")
 def test_gemv_wait_that_runs_out_is_reported_and_later_calls_are_right(tvl, shape):
     # CTA 0's last stage is never copied: its consumer gives up after the

@@ -13,8 +13,8 @@ torch = pytest.importorskip("torch")
 
 # split along K (S > 1), one row per CTA or more (S = 1), ragged and
 # unaligned-K shapes that take the per-row kernel
-SHAPES = [(768, 768), (2048, 768), (768, 2048), (5, 4096), (300, 288), (4096, 11008),
-          (32000, 768), (7, 13), (33, 4097)]
+SHAPES = [(768, 768), (2048, 768), (768, 2048), (5, 4096), (64, 8192), (100, 2048),
+          (300, 288), (4096, 11008), (32000, 768), (7, 13), (33, 4097)]
 
 
 @pytest.fixture(scope="module")
@@ -53,7 +53,7 @@ def test_noalloc_allocates_no_device_memory(tvl):
     """After the first call on the device (the one-time setup), further calls
     leave the device's free memory and the library's allocation count as they
     were."""
-    M, K = 768, 768  # split along K: the static scratch is in use
+    M, K = 64, 8192  # fewer rows than SMs: split along K, the static scratch is in use
     W, x = synth.gemv_operands(M, K, 12)
     dW, dx = torch.from_numpy(W).cuda(), torch.from_numpy(x).cuda()
     y = torch.empty(M, device="cuda")
