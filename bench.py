@@ -68,6 +68,8 @@ def parse():
     ap.add_argument("--gemv-sweep", action="store_true", help="GEMV GB/s per shape instead")
     ap.add_argument("--hot", action="store_true",
                     help="with --gemv-sweep: one copy of W, so that W stays in L2 when it fits")
+    ap.add_argument("--prefill", type=int, default=0,
+                    help="time tvl_prefill of this many prompt tokens instead of decoding")
     ap.add_argument("--batch", type=int, default=1, choices=[1, 2, 3, 4],
                     help="sequences decoded together per launch (tvl_decode_greedy_batch)")
     return ap.parse_args()
@@ -441,6 +443,70 @@ def gemv_sweep(args):
           flush=True)
 
 
+def prefill_bench(args, cfg):
+    """tokens/s of tvl_prefill: a prompt of args.prefill seeded token ids
+    (uniform in [3, 31999]) from position 0, one call per step, K calls timed
+    with CUDA events after W warm-up calls. The products run on the tensor
+    cores; the roofline is theirs: algorithmic FLOPs (2 per weight per
+    position, plus the causal attention's 4 hd per query-key pair) per second,
+    and the tensor pipe's share of the measured bf16 peak for the three bf16
+    products each float32 product takes."""
+    import torch
+    from paper_2601_03324_gb300 import synth, tvl
+    torch.cuda.set_device(0)
+    n = int(args.prefill)
+    blob = synth.make_blob(cfg)
+    stream = torch.cuda.Stream()
+    model = tvl.Model(cfg, blob, stream=stream.cuda_stream)
+    info = model.info()
+    prompt = synth.uniform_ints(n, synth.LONG_CONTEXT_SEED, 1, 3, 31999)
+    host = np.empty(cfg["vocab_size"], dtype=np.float32)
+    model.prefill(prompt, 0, host)  # first call: allocations, bf16 parts of the weights
+    for _ in range(max(3, args.warmup)):
+        model.prefill(prompt, 0)
+    model.sync()
+    props = torch.cuda.get_device_properties(0)
+    uuid = getattr(props, "uuid", None)
+    uuid = f"GPU-{uuid}" if uuid and not str(uuid).startswith("GPU-") else (str(uuid) if uuid else None)
+    clocks = Clocks(0, uuid)
+    time.sleep(0.15)
+    t0 = time.time()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        model.prefill(prompt, 0)
+    e1.record(stream)
+    model.sync()
+    clk = clocks.stop(t0, time.time())
+    ms = e0.elapsed_time(e1) / args.steps
+    d, F, L = cfg["dim"], cfg["hidden_dim"], cfg["n_layers"]
+    kvd = cfg["n_kv_heads"] * (d // cfg["n_heads"])
+    hd = d // cfg["n_heads"]
+    w_layers = L * ((d + 2 * kvd) * d + d * d + 3 * F * d)
+    flops = 2.0 * n * w_layers + 4.0 * hd * cfg["n_heads"] * L * n * (n + 1) / 2 + 2.0 * cfg["vocab_size"] * d
+    achieved = flops / (ms * 1e-3) / 1e12
+    pk = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))) if os.path.exists(
+        os.path.join(ROOT, "MEASURED_PEAKS.json")) else {}
+    bf16 = float(pk.get("bf16_tflops", 1900.0))
+    line = {"metric": f"prefill tokens/s ({args.workload}, {n}-token prompt, FP32 accuracy)",
+            "value": n / (ms * 1e-3), "unit": "tokens/s", "n_gpus": 1, "steps": args.steps,
+            "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True,
+            "dtype": "f32 (bf16 parts, fp32 accumulation)", "data": "synthetic (seeded N(0, 0.02) weights)",
+            "config": {"workload": args.workload, "prompt_tokens": n, "weights_seed": cfg["seed"],
+                       "l2": l2_statement(streamed_bytes_of(cfg))},
+            "roofline": {"bound": "tensor", "achieved": achieved, "unit": "TFLOP/s",
+                         "algorithmic_flops_per_call": flops,
+                         "tensor_pipe_frac": 3 * 2.0 * n * w_layers / (ms * 1e-3) / 1e12 / bf16,
+                         "peak_bf16": bf16,
+                         "note": "achieved = float32-equivalent FLOPs per second; the tensor "
+                                 "pipe runs three bf16 products for each (tensor_pipe_frac: "
+                                 "their share of the measured bf16 peak)"},
+            "clocks": clk, "grid": info.grid}
+    print(json.dumps(line), flush=True)
+    model.close()
+    return 0
+
+
 def main():
     args = parse()
     if args.weights == "q4" and not args.gemv_sweep:
@@ -456,6 +522,8 @@ def main():
     import torch.distributed as dist
     if args.gemv_sweep:
         return gemv_sweep(args)
+    if args.prefill:
+        return prefill_bench(args, cfg)
     if world > 1:
         dist.init_process_group("nccl", init_method="env://")
     torch.cuda.set_device(local_rank)
@@ -492,7 +560,8 @@ def main():
         model.sync()
         pms = pe0.elapsed_time(pe1) / 3
         prefill = {"tokens": len(prompt), "ms": pms, "tokens_per_s": len(prompt) / pms * 1e3,
-                   "note": "tvl_prefill of the prompt (cuBLAS float32 GEMMs per layer), "
+                   "note": "tvl_prefill of the prompt (tensor-core GEMMs in float32 accuracy "
+                           "per layer), "
                            "mean of 3 calls"}
         tok0, pos0 = int(np.argmax(host)), len(prompt)
         seq = cfg["max_seq"] - pos0

@@ -144,10 +144,13 @@ tvl_status tvl_decode_greedy_batch(tvl_model* m, int32_t batch, const int32_t* s
  * block of n rows per layer, writing their K/V rows into the cache, and the
  * logits of the last position are returned — the same computation as n
  * tvl_forward calls (§2.1, §7.1), with each layer's weights read once for all
- * n positions. The products with the weight matrices run as float32 GEMMs in
- * cuBLAS; the first call allocates the activations for max_seq positions
- * (and a cuBLAS handle), kept until tvl_free. Positions 0 .. start_pos - 1
- * must hold this sequence's K/V already.
+ * n positions. The products with the weight matrices run on the tensor
+ * cores in float32 accuracy (as tvl_gemm: bf16 parts, fp32 accumulation);
+ * the first call allocates the activations for max_seq positions and the
+ * bf16 parts of every layer's weight matrices (as many bytes as those
+ * float32 matrices: 340 MB at 110M, 26 GB at 7B), kept until tvl_free; a
+ * bounded wait that runs out in a product is reported by tvl_gemm_status.
+ * Positions 0 .. start_pos - 1 must hold this sequence's K/V already.
  *   logits_out: V floats, as for tvl_forward (device: no wait; host: waits;
  *   NULL: kept on the device).
  *   n >= 1, start_pos >= 0, start_pos + n <= max_seq, tokens in [0, V), else
@@ -168,6 +171,24 @@ tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n, int32_t s
  * reads x, writes y and copies W only once that kernel has completed. */
 tvl_status tvl_gemv(const float* W, const float* x, float* y, int32_t d_out, int32_t d_in,
                     void* stream);
+
+/* Y = X W^T for a block of n vectors (the products of a multi-token prefill,
+ * §2.1 and §7.1: n decode steps whose weight reads are shared), on the
+ * tensor cores (tcgen05) in float32 accuracy: each float is split into two
+ * bf16 parts (hi = bf16(a), lo = bf16(a - hi)) and the three products
+ * hi*hi + hi*lo + lo*hi are accumulated in fp32; what is dropped is about
+ * 2^-16 of each product. W [M x K], X [n x K], Y [n x M], row-major float32,
+ * device pointers, 16-byte aligned; K % 8 == 0 (else TVL_E_UNSUPPORTED);
+ * n, M, K >= 1 (else TVL_E_INVAL). Queued on `stream`, does not wait. A
+ * per-stream scratch buffer for the bf16 parts (4 (M + n) K bytes) is
+ * allocated on first use and grown when needed, kept until exit. */
+tvl_status tvl_gemm(const float* W, const float* X, float* Y, int32_t n, int32_t M, int32_t K,
+                    void* stream);
+
+/* Waits for `stream`, then reports (and clears) the tensor-core GEMM's error
+ * word: TVL_E_TIMEOUT if a bounded wait inside a tvl_gemm or prefill product
+ * ran out since the last query (that call's Y is incomplete), else TVL_OK. */
+tvl_status tvl_gemm_status(void* stream);
 
 /* Weight-only 8-bit rows (also the weight format of a model loaded with
  * weight_bits = 8). The paper leaves quantization to future work

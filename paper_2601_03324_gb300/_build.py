@@ -16,7 +16,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 OUT = os.path.join(HERE, "libtvl.so")
 BUILD_DIR = os.path.join(HERE, "_build")
-SOURCES = ["abi.cu", "decode.cu", "decode_batch.cu", "gemv.cu", "prefill.cu"]
+SOURCES = ["abi.cu", "decode.cu", "decode_batch.cu", "gemv.cu", "gemm.cu", "prefill.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -63,7 +63,7 @@ def build(force: bool = False, verbose: bool = False, extra: list[str] | None = 
         objs = list(ex.map(compile_one, SOURCES))
     tmp = OUT + ".tmp"
     cuda_lib = os.path.join(os.path.dirname(os.path.dirname(cc)), "lib64")
-    cmd = [cc, *ARCH, "-shared", "-o", tmp, *objs, "-lcublas",
+    cmd = [cc, *ARCH, "-shared", "-o", tmp, *objs,
            "-Xlinker", "-rpath", "-Xlinker", cuda_lib]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:

@@ -36,9 +36,9 @@ struct tvl_model {
   size_t xchg_off = 0, xchg_bytes = 0;
   tvl_status sticky = TVL_OK;
   // multi-token prefill (prefill.cu): created on first use
-  void* blas = nullptr;  // cublasHandle_t bound to `stream`
-  float* pf = nullptr;   // activations of up to max_seq positions
+  float* pf = nullptr;          // activations of up to max_seq positions
   size_t pf_bytes = 0;
+  unsigned char* pf_w = nullptr;  // bf16 parts of every layer's weight matrices
 };
 
 // Releases what prefill created (prefill.cu).

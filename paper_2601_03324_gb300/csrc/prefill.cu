@@ -4,15 +4,17 @@
 // logits come out. It is the same computation as n decode steps (paper §2.1
 // and §7.1 define the step; here the positions of a prompt share each layer's
 // weight reads), so its results equal n tvl_forward calls up to float
-// rounding. The products with the weight matrices are plain GEMMs
-// ([n x K] times [K x M]) and go to cuBLAS SGEMM in float32; the rest —
-// embedding rows, RMSNorm, RoPE and the cache write, causal attention, SwiGLU,
-// the residual adds — are the kernels below.
-#include <cublas_v2.h>
-
+// rounding. The products with the weight matrices ([n x K] times [K x M])
+// run on the tensor cores (gemm.cu: tcgen05, bf16 parts of every float, fp32
+// accumulation, float32 accuracy); the bf16 parts of the weights are made
+// once, at the first call. The rest — embedding rows, RMSNorm, RoPE and the
+// cache write, causal attention, SwiGLU, the residual adds — are the kernels
+// below, and the classifier row of the last position is the library's
+// streaming GEMV.
 #include <cmath>
 #include <string>
 
+#include "gemm.h"
 #include "model.h"
 
 using namespace tvl;
@@ -175,23 +177,20 @@ __global__ void swiglu_rows_kernel(const float* __restrict__ h13, float* __restr
   }
 }
 
-tvl_status blas_fail(cublasStatus_t s, const char* what) {
-  set_error(std::string(what) + " failed (cuBLAS status " + std::to_string((int)s) + ")");
-  return TVL_E_CUDA;
-}
+// The bf16 parts (hi then lo) of one weight matrix [M x K] in the prefill's
+// weight copy.
+struct Parts {
+  const unsigned char* hi;
+  const unsigned char* lo;
+};
 
-#define TVL_BLAS(call)                                  \
-  do {                                                  \
-    cublasStatus_t s_ = (call);                         \
-    if (s_ != CUBLAS_STATUS_SUCCESS) return blas_fail(s_, #call); \
-  } while (0)
-
-// Y[rows x M] = X[rows x K] W^T, W row-major [M x K], everything row-major.
-tvl_status gemm_rows(cublasHandle_t h, const float* W, const float* X, float* Y, int rows, int M,
-                     int K) {
-  const float one = 1.f, zero = 0.f;
-  TVL_BLAS(cublasSgemm(h, CUBLAS_OP_T, CUBLAS_OP_N, M, rows, K, &one, W, K, X, K, &zero, Y, M));
-  return TVL_OK;
+// Y[rows x M] = X[rows x K] W^T (everything row-major): X is split into its
+// bf16 parts (xh, xl) first, then the tensor-core GEMM.
+tvl_status gemm_rows(const Parts& w, const float* X, void* xh, void* xl, float* Y, int rows,
+                     int M, int K, int* err, cudaStream_t st) {
+  tvl_status s = split_bf16(X, xh, xl, (long long)rows * K, st);
+  if (s != TVL_OK) return s;
+  return gemm_bf16x3(w.hi, w.lo, xh, xl, Y, rows, M, K, M, err, st);
 }
 
 bool on_device(const void* p) {
@@ -206,10 +205,10 @@ bool on_device(const void* p) {
 }  // namespace
 
 void prefill_release(tvl_model* m) {
-  if (m->blas) cublasDestroy(static_cast<cublasHandle_t>(m->blas));
   lib_free(m->pf);
-  m->blas = nullptr;
+  lib_free(m->pf_w);
   m->pf = nullptr;
+  m->pf_w = nullptr;
   m->pf_bytes = 0;
 }
 
@@ -237,23 +236,45 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
   const DecodeArgs& a = m->args;
   const int d = a.d, F = a.F, kvd = a.kvd, hd = a.hd, S = a.S, L = a.L, V = a.V;
   cudaStream_t st = m->stream;
+  auto al = [](size_t b) { return (b + 255) / 256 * 256; };
+  // bf16 parts (hi, lo) of every layer's [Wq|Wk|Wv], Wo, W1/W3 (rows
+  // interleaved as in the arena, gains folded in) and W2, made at the first call
+  const size_t pq = al(2ull * (d + 2 * kvd) * d), po = al(2ull * d * d), p13 = al(4ull * F * d),
+               p2 = al(2ull * d * F);
+  const size_t per_layer = 2 * (pq + po + p13 + p2);
+  auto wsrc = [&](int l, int k) {  // the float32 matrix k of layer l in the arena
+    const unsigned char* lw = a.layer0 + (size_t)l * a.layer_stride;
+    return reinterpret_cast<const float*>(
+        lw + (k == 0 ? a.o_wqkv : k == 1 ? a.o_wo : k == 2 ? a.o_w13 : a.o_w2));
+  };
+  const size_t part_off[4] = {0, 2 * pq, 2 * pq + 2 * po, 2 * pq + 2 * po + 2 * p13};
+  const size_t part_len[4] = {pq, po, p13, p2};
+  const long long part_count[4] = {(long long)(d + 2 * kvd) * d, (long long)d * d,
+                                   2LL * F * d, (long long)d * F};
+  auto wparts = [&](int l, int k) {
+    const unsigned char* base = m->pf_w + (size_t)l * per_layer + part_off[k];
+    return Parts{base, base + part_len[k]};
+  };
+  if (!m->pf_w && L > 0) {
+    TVL_CK(lib_malloc((void**)&m->pf_w, per_layer * L));
+    for (int l = 0; l < L; ++l)
+      for (int k = 0; k < 4; ++k) {
+        const Parts p = wparts(l, k);
+        tvl_status s2 = split_bf16(wsrc(l, k), const_cast<unsigned char*>(p.hi),
+                                   const_cast<unsigned char*>(p.lo), part_count[k], st);
+        if (s2 != TVL_OK) return s2;
+      }
+  }
   // activations of up to S rows: x, x_b, qkv, att, h13, h; the last row's
-  // normalised vector; the tokens
+  // normalised vector; the tokens; the bf16 parts of a GEMM input
   const size_t fx = (size_t)S * d, fqkv = (size_t)S * (d + 2 * kvd), fh13 = (size_t)S * 2 * F,
                fh = (size_t)S * F;
-  const size_t need = 4 * (3 * fx + fqkv + fh13 + fh + d) + 4 * (size_t)S + 256;
+  const size_t xpart = al(2ull * S * (d > F ? d : F));
+  const size_t need = al(4 * (3 * fx + fqkv + fh13 + fh + d) + 4 * (size_t)S) + 2 * xpart;
   if (!m->pf) {
     TVL_CK(lib_malloc((void**)&m->pf, need));
     m->pf_bytes = need;
   }
-  if (!m->blas) {
-    cublasHandle_t h = nullptr;
-    TVL_BLAS(cublasCreate(&h));
-    m->blas = h;
-    TVL_BLAS(cublasSetMathMode(h, CUBLAS_DEFAULT_MATH));  // float32 products and sums
-  }
-  cublasHandle_t bh = static_cast<cublasHandle_t>(m->blas);
-  TVL_BLAS(cublasSetStream(bh, st));
   float* X = m->pf;
   float* XB = X + fx;
   float* QKV = XB + fx;
@@ -262,6 +283,12 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
   float* Hh = H13 + fh13;
   float* XN = Hh + fh;
   int* tok = reinterpret_cast<int*>(XN + d);
+  unsigned char* xh = reinterpret_cast<unsigned char*>(m->pf) +
+                      al(4 * (3 * fx + fqkv + fh13 + fh + d) + 4 * (size_t)S);
+  unsigned char* xl = xh + xpart;
+  int* err = nullptr;
+  tvl_status s = gemm_error_word(&err);
+  if (s != TVL_OK) return s;
   TVL_CK(cudaMemcpyAsync(tok, tokens, 4ull * n, cudaMemcpyHostToDevice, st));
 
   embed_rows_kernel<<<n, kRowThreads, 0, st>>>(a.E, tok, X, d);
@@ -271,41 +298,36 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
     const unsigned char* lw = a.layer0 + (size_t)l * a.layer_stride;
     const float* g_att = a.gains_folded ? nullptr : reinterpret_cast<const float*>(lw + a.o_gatt);
     const float* g_ffn = a.gains_folded ? nullptr : reinterpret_cast<const float*>(lw + a.o_gffn);
-    const float* Wqkv = reinterpret_cast<const float*>(lw + a.o_wqkv);
-    const float* Wo = reinterpret_cast<const float*>(lw + a.o_wo);
-    const float* W13 = reinterpret_cast<const float*>(lw + a.o_w13);  // interleaved rows
-    const float* W2 = reinterpret_cast<const float*>(lw + a.o_w2);
     float* kc = a.kc + (size_t)l * S * kvd;
     float* vc = a.vc + (size_t)l * S * kvd;
     rmsnorm_rows_kernel<<<n, kRowThreads, 0, st>>>(X, pending, g_att, XB, 0, d, a.eps);
     TVL_CK(cudaGetLastError());
-    tvl_status s;
-    if ((s = gemm_rows(bh, Wqkv, XB, QKV, n, d + 2 * kvd, d)) != TVL_OK) return s;
+    if ((s = gemm_rows(wparts(l, 0), XB, xh, xl, QKV, n, d + 2 * kvd, d, err, st)) != TVL_OK)
+      return s;
     rope_kv_kernel<<<n, kRowThreads, 0, st>>>(QKV, a.rope, kc, vc, start_pos, d, kvd, hd);
     TVL_CK(cudaGetLastError());
     const int warps = n * a.H, wpb = kRowThreads / 32;
     attention_rows_kernel<<<(warps + wpb - 1) / wpb, kRowThreads, 0, st>>>(
         QKV, kc, vc, ATT, n, start_pos, d, kvd, hd, a.H, a.Hkv, a.att_scale);
     TVL_CK(cudaGetLastError());
-    if ((s = gemm_rows(bh, Wo, ATT, XB, n, d, d)) != TVL_OK) return s;  // XB = Wo o
+    // XB = Wo o
+    if ((s = gemm_rows(wparts(l, 1), ATT, xh, xl, XB, n, d, d, err, st)) != TVL_OK) return s;
     rmsnorm_rows_kernel<<<n, kRowThreads, 0, st>>>(X, XB, g_ffn, ATT, 0, d, a.eps);  // ATT = x_b
     TVL_CK(cudaGetLastError());
-    if ((s = gemm_rows(bh, W13, ATT, H13, n, 2 * F, d)) != TVL_OK) return s;
+    if ((s = gemm_rows(wparts(l, 2), ATT, xh, xl, H13, n, 2 * F, d, err, st)) != TVL_OK) return s;
     const long long tot = (long long)n * F;
     swiglu_rows_kernel<<<(int)std::min<long long>((tot + 255) / 256, 4096), 256, 0, st>>>(H13, Hh,
                                                                                         tot);
     TVL_CK(cudaGetLastError());
-    if ((s = gemm_rows(bh, W2, Hh, XB, n, d, F)) != TVL_OK) return s;  // XB = W2 h
+    // XB = W2 h
+    if ((s = gemm_rows(wparts(l, 3), Hh, xh, xl, XB, n, d, F, err, st)) != TVL_OK) return s;
     pending = XB;
   }
   // the last position: x += (last update), x_b = RMSNorm(x, g_final), logits = Wcls x_b
   rmsnorm_rows_kernel<<<1, kRowThreads, 0, st>>>(X, pending, a.final_gain_folded ? nullptr : a.g_final,
                                                   XN, n - 1, d, a.eps);
   TVL_CK(cudaGetLastError());
-  {
-    const float one = 1.f, zero = 0.f;
-    TVL_BLAS(cublasSgemv(bh, CUBLAS_OP_T, d, V, &one, a.Wcls, d, XN, 1, &zero, a.logits, 1));
-  }
+  if ((s = tvl_gemv(a.Wcls, XN, a.logits, V, d, st)) != TVL_OK) return s;
   if (!logits_out) return TVL_OK;
   const size_t bytes = (size_t)V * 4;
   if (on_device(logits_out)) {

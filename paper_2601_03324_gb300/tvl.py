@@ -86,6 +86,10 @@ def _load():
     L.tvl_gemv_q4.argtypes = [P, P, P, i32, i32, P]
     L.tvl_gemv_noalloc.restype = st
     L.tvl_gemv_noalloc.argtypes = [P, P, P, i32, i32, P]
+    L.tvl_gemm.restype = st
+    L.tvl_gemm.argtypes = [P, P, P, i32, i32, i32, P]
+    L.tvl_gemm_status.restype = st
+    L.tvl_gemm_status.argtypes = [P]
     L.tvl_gemv_status.restype = st
     L.tvl_gemv_status.argtypes = [P]
     L.tvl_selftest_gemv_timeout.restype = st
@@ -118,6 +122,7 @@ lib = _load()
 EXPORTED = ["tvl_blob_bytes", "tvl_load", "tvl_load_file", "tvl_forward", "tvl_decode_greedy",
             "tvl_forward_batch", "tvl_decode_greedy_batch", "tvl_prefill",
             "tvl_gemv", "tvl_gemv_noalloc", "tvl_gemv_status", "tvl_selftest_gemv_timeout",
+            "tvl_gemm", "tvl_gemm_status",
             "tvl_q8_bytes", "tvl_quantize_q8", "tvl_gemv_q8",
             "tvl_q4_bytes", "tvl_quantize_q4", "tvl_gemv_q4",
             "tvl_sync", "tvl_free", "tvl_status_string", "tvl_last_error",
@@ -172,6 +177,17 @@ def tvl_gemv_noalloc(W, x, y, d_out: int, d_in: int, stream: int = 0):
     _check(lib.tvl_gemv_noalloc(ctypes.c_void_p(_addr(W)), ctypes.c_void_p(_addr(x)),
                                 ctypes.c_void_p(_addr(y)), int(d_out), int(d_in),
                                 ctypes.c_void_p(int(stream))), "tvl_gemv_noalloc")
+
+
+def tvl_gemm(W, X, Y, n: int, M: int, K: int, stream: int = 0):
+    """Y [n x M] = X [n x K] W^T on the tensor cores; device addresses."""
+    _check(lib.tvl_gemm(ctypes.c_void_p(_addr(W)), ctypes.c_void_p(_addr(X)),
+                        ctypes.c_void_p(_addr(Y)), int(n), int(M), int(K),
+                        ctypes.c_void_p(int(stream))), "tvl_gemm")
+
+
+def tvl_gemm_status(stream: int = 0) -> int:
+    return lib.tvl_gemm_status(ctypes.c_void_p(stream))
 
 
 def tvl_gemv_status(stream: int = 0) -> int:
