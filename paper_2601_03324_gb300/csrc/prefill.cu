@@ -166,6 +166,143 @@ __global__ void attention_rows_kernel(const float* __restrict__ qkv, const float
   }
 }
 
+// Causal attention of a block of queries, tiled (§2.1; the same arithmetic as
+// the per-row kernel above, in another order): one CTA of 128 threads takes 32
+// consecutive query rows of one head and walks the keys 0 .. (its last
+// position) in tiles of 32, with the Q, K and V tiles in shared memory (rows
+// padded by 4 floats, so that the float4 reads below hit distinct banks).
+// Thread (q, sub) = (tid / 4, tid % 4) scores keys sub, sub + 4, ..., sub + 28
+// of each tile for query q, the four threads of a query share an online
+// softmax (running max and sum, shuffles), and each accumulates its quarter of
+// the output row: float4 chunks sub, sub + 4, ... of the head's dims. kDpt =
+// head_dim / 4 (4 to 32, a multiple of 4).
+constexpr int kAttBQ = 32, kAttBK = 32, kAttThreads = 128;
+
+template <int kDpt>
+__global__ void __launch_bounds__(kAttThreads)
+    attention_tiles_kernel(const float* __restrict__ qkv, const float* __restrict__ kc,
+                           const float* __restrict__ vc, float* __restrict__ att, int n, int start,
+                           int d, int kvd, int H, int Hkv, float scale) {
+  constexpr int hd = 4 * kDpt, hp = hd + 4, hd4 = kDpt, nc = kDpt / 4;
+  extern __shared__ float sm[];
+  float* Qs = sm;                  // [BQ][hp], scaled by 1/sqrt(hd)
+  float* Ks = Qs + kAttBQ * hp;    // [BK][hp]
+  float* Vs = Ks + kAttBK * hp;    // [BK][hp]
+  float* Ps = Vs + kAttBK * hp;    // [BQ][BK + 1]
+  const int h = blockIdx.y, kvh = h / (H / Hkv);
+  const int i0 = blockIdx.x * kAttBQ;
+  const int tid = threadIdx.x, q = tid >> 2, sub = tid & 3;
+  const size_t rowlen = (size_t)d + 2 * kvd;
+  for (int e = tid; e < kAttBQ * hd4; e += kAttThreads) {
+    const int r = e / hd4, c = e - r * hd4;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (i0 + r < n) v = reinterpret_cast<const float4*>(qkv + (size_t)(i0 + r) * rowlen + h * hd)[c];
+    v.x *= scale;
+    v.y *= scale;
+    v.z *= scale;
+    v.w *= scale;
+    reinterpret_cast<float4*>(Qs + r * hp)[c] = v;
+  }
+  const int qpos = start + i0 + q;
+  const int last = min(start + i0 + kAttBQ - 1, start + n - 1);  // the tile's last position
+  float m = -INFINITY, l = 0.f;
+  float4 o[nc];
+#pragma unroll
+  for (int c = 0; c < nc; ++c) o[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int t0 = 0; t0 <= last; t0 += kAttBK) {
+    __syncthreads();  // the previous tile's K, V and P are read
+    for (int e = tid; e < kAttBK * hd4; e += kAttThreads) {
+      const int r = e / hd4, c = e - r * hd4, t = t0 + r;
+      float4 kv = make_float4(0.f, 0.f, 0.f, 0.f), vv = kv;
+      if (t <= last) {
+        kv = reinterpret_cast<const float4*>(kc + (size_t)t * kvd + kvh * hd)[c];
+        vv = reinterpret_cast<const float4*>(vc + (size_t)t * kvd + kvh * hd)[c];
+      }
+      reinterpret_cast<float4*>(Ks + r * hp)[c] = kv;
+      reinterpret_cast<float4*>(Vs + r * hp)[c] = vv;
+    }
+    __syncthreads();
+    float s[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) s[j] = 0.f;
+#pragma unroll 4
+    for (int c = 0; c < hd4; ++c) {
+      const float4 qv = reinterpret_cast<const float4*>(Qs + q * hp)[c];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float4 kv = reinterpret_cast<const float4*>(Ks + (sub + 4 * j) * hp)[c];
+        s[j] = fmaf(qv.x, kv.x, fmaf(qv.y, kv.y, fmaf(qv.z, kv.z, fmaf(qv.w, kv.w, s[j]))));
+      }
+    }
+    float mt = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      if (t0 + sub + 4 * j > qpos) s[j] = -INFINITY;  // causal: keys after the query
+      mt = fmaxf(mt, s[j]);
+    }
+    mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 1));
+    mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 2));
+    // key 0 is in the first tile for every query, so m is finite from then on
+    const float mn = fmaxf(m, mt);
+    const float corr = expf(m - mn);
+    float ps = 0.f;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      s[j] = expf(s[j] - mn);
+      ps += s[j];
+    }
+    ps += __shfl_xor_sync(0xffffffffu, ps, 1);
+    ps += __shfl_xor_sync(0xffffffffu, ps, 2);
+    l = l * corr + ps;
+    m = mn;
+#pragma unroll
+    for (int c = 0; c < nc; ++c) {
+      o[c].x *= corr;
+      o[c].y *= corr;
+      o[c].z *= corr;
+      o[c].w *= corr;
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) Ps[q * (kAttBK + 1) + sub + 4 * j] = s[j];
+    __syncwarp();  // the four threads of a query are lanes of one warp
+#pragma unroll 4
+    for (int k = 0; k < kAttBK; ++k) {
+      const float p = Ps[q * (kAttBK + 1) + k];
+      const float4* vr = reinterpret_cast<const float4*>(Vs + k * hp);
+#pragma unroll
+      for (int c = 0; c < nc; ++c) {
+        const float4 v = vr[4 * c + sub];
+        o[c].x = fmaf(p, v.x, o[c].x);
+        o[c].y = fmaf(p, v.y, o[c].y);
+        o[c].z = fmaf(p, v.z, o[c].z);
+        o[c].w = fmaf(p, v.w, o[c].w);
+      }
+    }
+  }
+  if (i0 + q < n) {
+    const float inv = 1.0f / l;
+    float4* out = reinterpret_cast<float4*>(att + (size_t)(i0 + q) * d + h * hd);
+#pragma unroll
+    for (int c = 0; c < nc; ++c)
+      out[4 * c + sub] = make_float4(o[c].x * inv, o[c].y * inv, o[c].z * inv, o[c].w * inv);
+  }
+}
+
+template <int kDpt>
+tvl_status launch_attention_tiles(const float* qkv, const float* kc, const float* vc, float* att,
+                                  int n, int start, int d, int kvd, int H, int Hkv, float scale,
+                                  cudaStream_t st) {
+  constexpr int hp = 4 * kDpt + 4;
+  const int smem = (int)(sizeof(float) * ((kAttBQ + 2 * kAttBK) * hp + kAttBQ * (kAttBK + 1)));
+  TVL_CK(cudaFuncSetAttribute((const void*)attention_tiles_kernel<kDpt>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+  const dim3 grid((n + kAttBQ - 1) / kAttBQ, H);
+  attention_tiles_kernel<kDpt><<<grid, kAttThreads, smem, st>>>(qkv, kc, vc, att, n, start, d,
+                                                                kvd, H, Hkv, scale);
+  TVL_CK(cudaGetLastError());
+  return TVL_OK;
+}
+
 // h[i][j] = silu(a) * b with (a, b) = rows (2j, 2j + 1) of the interleaved
 // W1/W3 output (§2.1, SwiGLU).
 __global__ void swiglu_rows_kernel(const float* __restrict__ h13, float* __restrict__ h,
@@ -306,10 +443,27 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
       return s;
     rope_kv_kernel<<<n, kRowThreads, 0, st>>>(QKV, a.rope, kc, vc, start_pos, d, kvd, hd);
     TVL_CK(cudaGetLastError());
-    const int warps = n * a.H, wpb = kRowThreads / 32;
-    attention_rows_kernel<<<(warps + wpb - 1) / wpb, kRowThreads, 0, st>>>(
-        QKV, kc, vc, ATT, n, start_pos, d, kvd, hd, a.H, a.Hkv, a.att_scale);
-    TVL_CK(cudaGetLastError());
+    {  // head dims of 16 to 128 in steps of 16 take the tiled kernel
+      const float sc = a.att_scale;
+      s = TVL_OK;
+      switch (hd) {
+        case 16: s = launch_attention_tiles<4>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
+        case 32: s = launch_attention_tiles<8>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
+        case 48: s = launch_attention_tiles<12>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
+        case 64: s = launch_attention_tiles<16>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
+        case 80: s = launch_attention_tiles<20>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
+        case 96: s = launch_attention_tiles<24>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
+        case 112: s = launch_attention_tiles<28>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
+        case 128: s = launch_attention_tiles<32>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
+        default: {
+          const int warps = n * a.H, wpb = kRowThreads / 32;
+          attention_rows_kernel<<<(warps + wpb - 1) / wpb, kRowThreads, 0, st>>>(
+              QKV, kc, vc, ATT, n, start_pos, d, kvd, hd, a.H, a.Hkv, a.att_scale);
+          TVL_CK(cudaGetLastError());
+        }
+      }
+      if (s != TVL_OK) return s;
+    }
     // XB = Wo o
     if ((s = gemm_rows(wparts(l, 1), ATT, xh, xl, XB, n, d, d, err, st)) != TVL_OK) return s;
     rmsnorm_rows_kernel<<<n, kRowThreads, 0, st>>>(X, XB, g_ffn, ATT, 0, d, a.eps);  // ATT = x_b
