@@ -42,7 +42,7 @@ constexpr int kMaxBatch = 4;        // sequences one launch can decode together
 // reduction scratch (floats 8..39, ints 80..87), the five stage plans.
 constexpr int kPlansOffset = 512;
 constexpr int kMiscBytes = 1024;
-constexpr uint32_t kRefillDelayNs = 1000;  // producer pause before refilling freed stages
+constexpr uint32_t kRefillDelayNs = 0;  // producer pause before refilling freed stages (measured best: 0, with the L2 prefetch)
 
 struct DecodeArgs {
   // weights (inside the arena)

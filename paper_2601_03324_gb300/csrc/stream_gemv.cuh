@@ -84,6 +84,9 @@ __host__ __device__ inline StagePlan plan_stages(long long M, int K, int G, int 
     if (spread < 1) spread = 1;
     if (gran == 2) spread += spread & 1;
     p.rps = spread < cap ? spread : cap;
+    // more than four rows: whole passes of four (the row routine takes up to
+    // four rows at once, and a pass of one row costs a full warp reduction)
+    if (p.rps > 4) p.rps &= ~3;
     if (gran == 2 && p.rps >= 2) p.rps &= ~1;
     p.defer = gran == 2 && p.rps < 2;
     p.spr = 1;
