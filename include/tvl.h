@@ -146,7 +146,9 @@ tvl_status tvl_decode_greedy_batch(tvl_model* m, int32_t batch, const int32_t* s
  * tvl_forward calls (§2.1, §7.1), with each layer's weights read once for all
  * n positions. The products with the weight matrices run on the tensor
  * cores in float32 accuracy (as tvl_gemm: bf16 parts, fp32 accumulation);
- * the first call allocates the activations for max_seq positions and the
+ * the first call allocates the activations for max_seq positions (with the
+ * partial sums of up to eight key ranges per query and head of the
+ * attention, 4 * 8 * max_seq * H * (head_dim + 4) bytes) and the
  * bf16 parts of every layer's weight matrices (as many bytes as those
  * float32 matrices: 340 MB at 110M, 26 GB at 7B), kept until tvl_free; a
  * bounded wait that runs out in a product is reported by tvl_gemm_status.

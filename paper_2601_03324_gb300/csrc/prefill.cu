@@ -168,8 +168,11 @@ __global__ void attention_rows_kernel(const float* __restrict__ qkv, const float
 
 // Causal attention of a block of queries, tiled (§2.1; the same arithmetic as
 // the per-row kernel above, in another order): one CTA of 128 threads takes 32
-// consecutive query rows of one head and walks the keys 0 .. (its last
-// position) in tiles of 32, with the Q, K and V tiles in shared memory (rows
+// consecutive query rows of one head and walks its share of the keys
+// 0 .. (its last position) in tiles of 32 (split z of the key range:
+// tiles [z T, (z + 1) T); with more than one split each CTA writes its rows'
+// unnormalised partials (o, max, sum) to `part` and attention_merge_kernel
+// combines them), with the Q, K and V tiles in shared memory (rows
 // padded by 4 floats, so that the float4 reads below hit distinct banks).
 // Thread (q, sub) = (tid / 4, tid % 4) scores keys sub, sub + 4, ..., sub + 28
 // of each tile for query q, the four threads of a query share an online
@@ -177,12 +180,14 @@ __global__ void attention_rows_kernel(const float* __restrict__ qkv, const float
 // the output row: float4 chunks sub, sub + 4, ... of the head's dims. kDpt =
 // head_dim / 4 (4 to 32, a multiple of 4).
 constexpr int kAttBQ = 32, kAttBK = 32, kAttThreads = 128;
+constexpr int kAttSplits = 8;  // key splits of the longest rows, at most
 
 template <int kDpt>
 __global__ void __launch_bounds__(kAttThreads)
     attention_tiles_kernel(const float* __restrict__ qkv, const float* __restrict__ kc,
                            const float* __restrict__ vc, float* __restrict__ att, int n, int start,
-                           int d, int kvd, int H, int Hkv, float scale) {
+                           int d, int kvd, int H, int Hkv, float scale, int tiles_per_split,
+                           float* __restrict__ part) {
   constexpr int hd = 4 * kDpt, hp = hd + 4, hd4 = kDpt, nc = kDpt / 4;
   extern __shared__ float sm[];
   float* Qs = sm;                  // [BQ][hp], scaled by 1/sqrt(hd)
@@ -193,6 +198,10 @@ __global__ void __launch_bounds__(kAttThreads)
   const int i0 = blockIdx.x * kAttBQ;
   const int tid = threadIdx.x, q = tid >> 2, sub = tid & 3;
   const size_t rowlen = (size_t)d + 2 * kvd;
+  const int last = min(start + i0 + kAttBQ - 1, start + n - 1);  // the tile's last position
+  const int k_begin = blockIdx.z * tiles_per_split * kAttBK;
+  if (k_begin > last) return;  // this split holds no key of these rows (uniform in the CTA)
+  const int k_end = min(last, k_begin + tiles_per_split * kAttBK - 1);
   for (int e = tid; e < kAttBQ * hd4; e += kAttThreads) {
     const int r = e / hd4, c = e - r * hd4;
     float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -204,17 +213,16 @@ __global__ void __launch_bounds__(kAttThreads)
     reinterpret_cast<float4*>(Qs + r * hp)[c] = v;
   }
   const int qpos = start + i0 + q;
-  const int last = min(start + i0 + kAttBQ - 1, start + n - 1);  // the tile's last position
   float m = -INFINITY, l = 0.f;
   float4 o[nc];
 #pragma unroll
   for (int c = 0; c < nc; ++c) o[c] = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int t0 = 0; t0 <= last; t0 += kAttBK) {
+  for (int t0 = k_begin; t0 <= k_end; t0 += kAttBK) {
     __syncthreads();  // the previous tile's K, V and P are read
     for (int e = tid; e < kAttBK * hd4; e += kAttThreads) {
       const int r = e / hd4, c = e - r * hd4, t = t0 + r;
       float4 kv = make_float4(0.f, 0.f, 0.f, 0.f), vv = kv;
-      if (t <= last) {
+      if (t <= k_end) {
         kv = reinterpret_cast<const float4*>(kc + (size_t)t * kvd + kvh * hd)[c];
         vv = reinterpret_cast<const float4*>(vc + (size_t)t * kvd + kvh * hd)[c];
       }
@@ -242,13 +250,15 @@ __global__ void __launch_bounds__(kAttThreads)
     }
     mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 1));
     mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 2));
-    // key 0 is in the first tile for every query, so m is finite from then on
+    // a query whose keys so far in this split are all after it has no
+    // maximum yet (mn = -inf): nothing to add and nothing to rescale
     const float mn = fmaxf(m, mt);
-    const float corr = expf(m - mn);
+    const bool none = mn == -INFINITY;
+    const float corr = none ? 1.f : expf(m - mn);
     float ps = 0.f;
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      s[j] = expf(s[j] - mn);
+      s[j] = none ? 0.f : expf(s[j] - mn);
       ps += s[j];
     }
     ps += __shfl_xor_sync(0xffffffffu, ps, 1);
@@ -280,26 +290,82 @@ __global__ void __launch_bounds__(kAttThreads)
     }
   }
   if (i0 + q < n) {
-    const float inv = 1.0f / l;
-    float4* out = reinterpret_cast<float4*>(att + (size_t)(i0 + q) * d + h * hd);
+    if (part) {  // partial of split z: o (unnormalised), then max and sum
+      float* pr = part + (((size_t)blockIdx.z * n + i0 + q) * H + h) * (hd + 4);
+      float4* out = reinterpret_cast<float4*>(pr);
 #pragma unroll
-    for (int c = 0; c < nc; ++c)
-      out[4 * c + sub] = make_float4(o[c].x * inv, o[c].y * inv, o[c].z * inv, o[c].w * inv);
+      for (int c = 0; c < nc; ++c) out[4 * c + sub] = o[c];
+      if (sub == 0) {
+        pr[hd] = m;
+        pr[hd + 1] = l;
+      }
+    } else {
+      const float inv = 1.0f / l;
+      float4* out = reinterpret_cast<float4*>(att + (size_t)(i0 + q) * d + h * hd);
+#pragma unroll
+      for (int c = 0; c < nc; ++c)
+        out[4 * c + sub] = make_float4(o[c].x * inv, o[c].y * inv, o[c].z * inv, o[c].w * inv);
+    }
+  }
+}
+
+// Combines the key splits of attention_tiles_kernel, one warp per (row, head):
+// o = sum_z e^(m_z - M) o_z / sum_z e^(m_z - M) l_z, M = max_z m_z, over the
+// splits that hold keys of the row's 32-row block (split 0 holds key 0 of every
+// row, so M is finite; a split with no key up to the row has m = -inf and
+// weight 0).
+__global__ void attention_merge_kernel(const float* __restrict__ part, float* __restrict__ att,
+                                       int n, int start, int d, int H, int hd,
+                                       int tiles_per_split) {
+  const int gw = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (gw >= n * H) return;
+  const int lane = threadIdx.x & 31, i = gw / H, h = gw - i * H;
+  const int last = min(start + (i / kAttBQ) * kAttBQ + kAttBQ - 1, start + n - 1);
+  const int nz = last / (tiles_per_split * kAttBK) + 1;
+  const size_t stride = (size_t)n * H * (hd + 4);
+  const float* p0 = part + ((size_t)i * H + h) * (hd + 4);
+  float M = -INFINITY;
+  for (int z = 0; z < nz; ++z) M = fmaxf(M, p0[z * stride + hd]);
+  float L = 0.f;
+  for (int z = 0; z < nz; ++z) {
+    const float mz = p0[z * stride + hd];
+    if (mz != -INFINITY) L += expf(mz - M) * p0[z * stride + hd + 1];
+  }
+  const float inv = 1.0f / L;
+  for (int j = lane; j < hd; j += 32) {
+    float o = 0.f;
+    for (int z = 0; z < nz; ++z) {
+      const float mz = p0[z * stride + hd];
+      if (mz != -INFINITY) o = fmaf(expf(mz - M), p0[z * stride + j], o);
+    }
+    att[(size_t)i * d + h * hd + j] = o * inv;
   }
 }
 
 template <int kDpt>
 tvl_status launch_attention_tiles(const float* qkv, const float* kc, const float* vc, float* att,
                                   int n, int start, int d, int kvd, int H, int Hkv, float scale,
-                                  cudaStream_t st) {
+                                  float* part, cudaStream_t st) {
   constexpr int hp = 4 * kDpt + 4;
   const int smem = (int)(sizeof(float) * ((kAttBQ + 2 * kAttBK) * hp + kAttBQ * (kAttBK + 1)));
   TVL_CK(cudaFuncSetAttribute((const void*)attention_tiles_kernel<kDpt>,
                               cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-  const dim3 grid((n + kAttBQ - 1) / kAttBQ, H);
-  attention_tiles_kernel<kDpt><<<grid, kAttThreads, smem, st>>>(qkv, kc, vc, att, n, start, d,
-                                                                kvd, H, Hkv, scale);
+  // split the key range of the longest rows over up to kAttSplits CTAs of at
+  // least four tiles each
+  const int ntiles = (start + n + kAttBK - 1) / kAttBK;
+  int tps = (ntiles + kAttSplits - 1) / kAttSplits;
+  if (tps < 4) tps = 4;
+  const int nsplit = (ntiles + tps - 1) / tps;
+  const dim3 grid((n + kAttBQ - 1) / kAttBQ, H, nsplit);
+  attention_tiles_kernel<kDpt><<<grid, kAttThreads, smem, st>>>(
+      qkv, kc, vc, att, n, start, d, kvd, H, Hkv, scale, tps, nsplit > 1 ? part : nullptr);
   TVL_CK(cudaGetLastError());
+  if (nsplit > 1) {
+    const int warps = n * H, wpb = kRowThreads / 32;
+    attention_merge_kernel<<<(warps + wpb - 1) / wpb, kRowThreads, 0, st>>>(part, att, n, start, d,
+                                                                           H, 4 * kDpt, tps);
+    TVL_CK(cudaGetLastError());
+  }
   return TVL_OK;
 }
 
@@ -407,7 +473,10 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
   const size_t fx = (size_t)S * d, fqkv = (size_t)S * (d + 2 * kvd), fh13 = (size_t)S * 2 * F,
                fh = (size_t)S * F;
   const size_t xpart = al(2ull * S * (d > F ? d : F));
-  const size_t need = al(4 * (3 * fx + fqkv + fh13 + fh + d) + 4 * (size_t)S) + 2 * xpart;
+  // partials (o, max, sum) of the attention's key splits
+  const size_t fpart = (size_t)kAttSplits * S * a.H * (hd + 4);
+  const size_t need = al(4 * (3 * fx + fqkv + fh13 + fh + d) + 4 * (size_t)S) + 2 * xpart +
+                      al(4 * fpart);
   if (!m->pf) {
     TVL_CK(lib_malloc((void**)&m->pf, need));
     m->pf_bytes = need;
@@ -423,6 +492,7 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
   unsigned char* xh = reinterpret_cast<unsigned char*>(m->pf) +
                       al(4 * (3 * fx + fqkv + fh13 + fh + d) + 4 * (size_t)S);
   unsigned char* xl = xh + xpart;
+  float* PART = reinterpret_cast<float*>(xl + xpart);
   int* err = nullptr;
   tvl_status s = gemm_error_word(&err);
   if (s != TVL_OK) return s;
@@ -447,14 +517,14 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
       const float sc = a.att_scale;
       s = TVL_OK;
       switch (hd) {
-        case 16: s = launch_attention_tiles<4>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
-        case 32: s = launch_attention_tiles<8>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
-        case 48: s = launch_attention_tiles<12>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
-        case 64: s = launch_attention_tiles<16>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
-        case 80: s = launch_attention_tiles<20>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
-        case 96: s = launch_attention_tiles<24>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
-        case 112: s = launch_attention_tiles<28>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
-        case 128: s = launch_attention_tiles<32>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, st); break;
+        case 16: s = launch_attention_tiles<4>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 32: s = launch_attention_tiles<8>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 48: s = launch_attention_tiles<12>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 64: s = launch_attention_tiles<16>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 80: s = launch_attention_tiles<20>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 96: s = launch_attention_tiles<24>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 112: s = launch_attention_tiles<28>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 128: s = launch_attention_tiles<32>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
         default: {
           const int warps = n * a.H, wpb = kRowThreads / 32;
           attention_rows_kernel<<<(warps + wpb - 1) / wpb, kRowThreads, 0, st>>>(

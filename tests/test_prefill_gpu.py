@@ -126,3 +126,35 @@ def test_110m_prefill_896_prompt_then_greedy(tvl):
         rtoks, rlg = ref.greedy(start, 32, start_pos=896)
         gen = m.decode_greedy(start, 896, 32)
         compare_greedy(gen, rtoks[1:] + [int(np.argmax(rlg[-1]))], rlg)
+
+
+@pytest.mark.parametrize("parts,kw", [
+    ((300, 140), dict()),                                     # 14 key tiles: 4 splits of 4
+    ((1050,), dict(dim=128, n_heads=2, n_kv_heads=1)),        # 33 tiles: 7 splits of 5, hd 64
+    ((129, 3, 700), dict(n_kv_heads=2)),                      # ragged parts, grouped heads
+], ids=["two_parts", "long_hd64", "ragged"])
+def test_prefill_long_key_ranges_split_across_ctas(tvl, parts, kw):
+    """Rows that see more than 128 keys have their key range cut into up to
+    eight parts, each a CTA of its own, whose partial sums are merged; the
+    logits after each part and the continuation (which reads every row's K/V
+    of the second layer, made from the first layer's merged attention) must
+    match the oracle."""
+    cfg = small_config(max_seq=1100, **kw)
+    V = cfg["vocab_size"]
+    blob = synth.make_blob(cfg, seed=45)
+    toks = synth.uniform_ints(sum(parts), 7, 0, 0, V - 1)
+    ref = oracle.Model(cfg, blob, 64)
+    out = np.empty(V, np.float32)
+    with tvl.Model(cfg, blob) as m:
+        p0 = 0
+        for n in parts:
+            m.prefill(toks[p0:p0 + n], p0, out)
+            lg = oracle_run(ref, toks[p0:p0 + n], p0)
+            assert_logits_close(out, lg, f"prefill {p0}..{p0 + n - 1}")
+            p0 += n
+        t = int(np.argmax(lg))
+        for s in range(4):
+            m.forward(t, p0 + s, out)
+            lg = ref.forward(t, p0 + s)
+            assert_logits_close(out, lg, f"decode pos {p0 + s}")
+            t = int(np.argmax(lg))
