@@ -341,7 +341,9 @@ int64_t tvl_debug_live_allocations(void);
  * next_tag), 1 .. 2^32 - 1, else TVL_E_INVAL. Tags are 32-bit and 0 marks a
  * word never written: a launch whose tags would pass 2^32 - 1 first zeroes
  * the exchange words on the model's stream and starts again from tag 1. This
- * hook puts a model next to that point without 2^32 exchanges of decoding. */
+ * hook puts a model next to that point without 2^32 exchanges of decoding.
+ * A tag below the model's next one also zeroes the exchange words first
+ * (queued on the model's stream), since published words only grow. */
 tvl_status tvl_debug_set_next_tag(tvl_model* m, uint64_t tag);
 
 #ifdef __cplusplus
