@@ -74,9 +74,9 @@ struct SmemPlan {
 
 // Shared memory of one CTA for B sequences: the ring takes what the other
 // regions leave, up to kMaxStages stages.
-SmemPlan plan_smem(int d, int F, int hd, int max_bytes, int B) {
+SmemPlan plan_smem(int d, int F, int hd, int nch_cap, int max_bytes, int B) {
   SmemPlan p{};
-  const int att_floats = 3 * hd + kAttMaxChunk + 4 * kConsumerThreads + 16;
+  const int att_floats = 3 * hd + kAttMaxChunk + 4 * kConsumerThreads + nch_cap * (hd + 2) + 16;
   // every region is a multiple of 128 bytes, so every region starts aligned
   const int xs = (int)a128(4LL * B * d), vec = (int)a128(4LL * B * std::max(d, F));
   const int seg = (int)a128(kMaxSegParts * 4), att = (int)a128(4LL * att_floats), misc = kMiscBytes;
@@ -269,7 +269,7 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   // a head gets the most attention chunks with one sequence: this bounds every B
   const int nch_cap = nch_cap_for(S, H, G);
   for (int B = 1; B <= maxB; ++B) {
-    const SmemPlan sp = plan_smem(d, F, hd, max_optin, B);
+    const SmemPlan sp = plan_smem(d, F, hd, nch_cap, max_optin, B);
     {  // segment partials of rows longer than a stage must fit the scratch
       const long long Ms[5] = {d + 2LL * kvd, d, 2LL * F, d, V};
       const int Ks[5] = {d, d, d, F, d};
@@ -345,6 +345,7 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   const size_t o_h13 = take(8ull * F * nB);
   const size_t o_f = take(8ull * d * nB), o_lg = take(4ull * V * nB);
   const size_t o_att = take(8ull * H * nch_cap * att_stride * nB);
+  const size_t o_attn = take(8ull * d * nB);
   const size_t o_cand = take(8ull * 2 * G * 2 * nB), o_tok = take(4ull * S * nB);
   const size_t o_ts = take(8ull * S), o_err = take(4);
   m->arena_bytes = off;
@@ -498,6 +499,7 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   a.x_f = reinterpret_cast<unsigned long long*>(m->arena + o_f);
   a.logits = reinterpret_cast<float*>(m->arena + o_lg);
   a.x_att = reinterpret_cast<unsigned long long*>(m->arena + o_att);
+  a.x_attn = reinterpret_cast<unsigned long long*>(m->arena + o_attn);
   a.x_cand = reinterpret_cast<unsigned long long*>(m->arena + o_cand);
   a.tokens = reinterpret_cast<int*>(m->arena + o_tok);
   a.ts = reinterpret_cast<unsigned long long*>(m->arena + o_ts);

@@ -63,7 +63,8 @@ struct DecodeArgs {
   float* vc;
   // tagged exchange buffers (64-bit words: tag << 32 | float bits)
   unsigned long long* x_qkv;   // [d + 2 kvd]
-  unsigned long long* x_att;   // [H][nch_cap][att_stride]: m, l, -, -, sum[hd] of every chunk
+  unsigned long long* x_att;   // [H][nch_cap][att_stride]: m, l, -, -, sum[hd] of chunks > 0
+  unsigned long long* x_attn;  // [d]: attention output, merged per head
   unsigned long long* x_o;     // [d]
   unsigned long long* x_h13;   // [F]: h = silu(W1 x_b) * (W3 x_b)
   unsigned long long* x_f;     // [d]
@@ -481,9 +482,13 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
   const int ppw = 32 / lpp;
   const int sub = lane / lpp, li = lane - sub * lpp;
 
+  // the items of chunk 0 (the heads' mergers) come after the other items of
+  // the same CTA, which they wait for
+  for (int pass = 0; pass < 2; ++pass)
   for (int it = blockIdx.x; it < kB * a.H * nch; it += a.G) {
     const int b = kB == 1 ? 0 : it / (a.H * nch), hc = it - b * a.H * nch;
     const int h = hc / nch, c = hc - h * nch;
+    if ((c == 0) != (pass == 1)) continue;
     const int kvh = h / group;
     const size_t lay = (size_t)b * a.kv_seq + (size_t)l * a.S * a.kvd;
     const unsigned long long* xq = a.x_qkv + (size_t)b * (a.d + 2 * a.kvd);
@@ -663,114 +668,47 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
     float own = 0.f;  // this chunk's sum of e_t v_t, element tid (tid < hd)
     if (tid < hd)
       for (int g2 = 0; g2 < ng; ++g2) own += part[g2 * hd + tid];
-    // the chunk's record; every CTA merges the records of all chunks (the new
-    // cache row is released later, off this path: see wrote_kv)
-    {
+    // the chunk's record (the new cache row is released later, off this
+    // path: see wrote_kv)
+    if (c != 0) {
       unsigned long long* rec = a.x_att + ((size_t)hb * a.nch_cap + c) * a.att_stride;
       if (tid < hd) st_tag(rec + 4 + tid, tag_att, own);
       if (tid == 0) {
         st_tag(rec, tag_att, m);
         st_tag(rec + 1, tag_att, ls);
       }
+    } else {
+      // the head's merger: records of chunks 1..nch-1 as pairs (m, l), (sum[2i], sum[2i+1]);
+      // o_h[j] = sum_c w_c sum_c[j], w_c = exp(m_c - M) / sum_c' exp(m_c' - M) l_c', chunk order
+      float* mrg = part + 4 * kConsumerThreads;  // [nch - 1][hd + 2]
+      const int ppr = 1 + half;
+      const bool ok2 = poll_pairs_at(
+          (nch - 1) * ppr,
+          [&](int p) {
+            const int cc = 1 + p / ppr, k = p - (cc - 1) * ppr;
+            const unsigned long long* r0 = a.x_att + ((size_t)hb * a.nch_cap + cc) * a.att_stride;
+            return k == 0 ? r0 : r0 + 4 + 2 * (k - 1);
+          },
+          tag_att, pc, [&](int p, float x0, float x1) {
+            const int cc = p / ppr, k = p - cc * ppr;
+            float* rr = mrg + cc * (hd + 2);
+            rr[k == 0 ? 0 : 2 * k] = x0;
+            rr[k == 0 ? 1 : 2 * k + 1] = x1;
+          });
+      if (!vote_ok(ok2, pc.s_abort)) return false;
+      if (tid < hd) {
+        float M = m;
+        for (int cc = 0; cc < nch - 1; ++cc) M = fmaxf(M, mrg[cc * (hd + 2)]);
+        float Lsum = expf(m - M) * ls;
+        for (int cc = 0; cc < nch - 1; ++cc)
+          Lsum += expf(mrg[cc * (hd + 2)] - M) * mrg[cc * (hd + 2) + 1];
+        float o = (expf(m - M) / Lsum) * own;
+        for (int cc = 0; cc < nch - 1; ++cc)
+          o = fmaf(expf(mrg[cc * (hd + 2)] - M) / Lsum, mrg[cc * (hd + 2) + 2 + tid], o);
+        st_tag(a.x_attn + (size_t)hb * hd + tid, tag_att, o);
+      }
     }
     named_bar_sync(kBarConsumers, kConsumerThreads);
-  }
-  return true;
-}
-
-// The attention output of every (sequence, head), merged into vec from the
-// records of its chunks (paper §2.1: one softmax over positions 0..pos, here
-// computed chunk by chunk). Chunk c published its largest score m_c, l_c =
-// sum_t e^(s_t - m_c) and s_c = sum_t e^(s_t - m_c) v_t; the output is
-// o = sum_c e^(m_c - M) s_c / sum_c e^(m_c - M) l_c with M = max_c m_c, folded
-// here chunk by chunk in chunk order (a new running maximum rescales what
-// was added before), so every CTA gets the same bits. Work item (sequence,
-// head, output pair q): its thread polls the (m, l) pair and output pair q of
-// every chunk of the head; each thread takes two items at a time, with
-// kMergeChunks chunks of both in flight.
-constexpr int kMergeChunks = 4;
-template <int kB>
-__device__ inline bool merge_records(const DecodeArgs& a, int pos, unsigned tag, float* vec,
-                                     int vs, const Poll& pc) {
-  int nch, clen;
-  att_split(pos, a.H * kB, a.G, &nch, &clen);
-  const int half = a.hd >> 1, nitems = kB * a.H * half;
-  const size_t hstride = (size_t)a.nch_cap * a.att_stride;  // words from one head's records to the next
-  for (int w0 = threadIdx.x; w0 < nitems; w0 += 2 * kConsumerThreads) {
-    int hb[2], q[2];
-    bool has[2];
-    float M[2], L[2], o0[2], o1[2];
-#pragma unroll
-    for (int i = 0; i < 2; ++i) {
-      const int w = w0 + i * kConsumerThreads;
-      has[i] = w < nitems;
-      const int ww = has[i] ? w : w0;
-      hb[i] = ww / half;  // sequence * H + head
-      q[i] = ww - hb[i] * half;
-      M[i] = -INFINITY;
-      L[i] = 0.f;
-      o0[i] = 0.f;
-      o1[i] = 0.f;
-    }
-    for (int c0 = 0; c0 < nch; c0 += kMergeChunks) {
-      ulonglong2 ml[2][kMergeChunks], sv[2][kMergeChunks];
-      unsigned pending = 0;
-#pragma unroll
-      for (int i = 0; i < 2; ++i)
-#pragma unroll
-        for (int j = 0; j < kMergeChunks; ++j)
-          if (has[i] && c0 + j < nch) {
-            const unsigned long long* r = a.x_att + hb[i] * hstride + (size_t)(c0 + j) * a.att_stride;
-            ml[i][j] = ld_tag2(r);
-            sv[i][j] = ld_tag2(r + 4 + 2 * q[i]);
-            pending |= 1u << (i * kMergeChunks + j);
-          }
-      PollClock clk;
-      while (true) {
-#pragma unroll
-        for (int i = 0; i < 2; ++i)
-#pragma unroll
-          for (int j = 0; j < kMergeChunks; ++j) {
-            const unsigned bit = 1u << (i * kMergeChunks + j);
-            if ((pending & bit) && tags_are(ml[i][j], tag) && tags_are(sv[i][j], tag))
-              pending &= ~bit;
-          }
-        if (!pending) break;
-        if (!clk.keep_waiting(pc)) return false;
-#pragma unroll
-        for (int i = 0; i < 2; ++i)
-#pragma unroll
-          for (int j = 0; j < kMergeChunks; ++j)
-            if ((pending >> (i * kMergeChunks + j)) & 1u) {
-              const unsigned long long* r =
-                  a.x_att + hb[i] * hstride + (size_t)(c0 + j) * a.att_stride;
-              ml[i][j] = ld_tag2(r);
-              sv[i][j] = ld_tag2(r + 4 + 2 * q[i]);
-            }
-      }
-#pragma unroll
-      for (int i = 0; i < 2; ++i)
-#pragma unroll
-        for (int j = 0; j < kMergeChunks; ++j)
-          if (has[i] && c0 + j < nch) {
-            const float mc = lo_f(ml[i][j].x), lc = lo_f(ml[i][j].y);
-            const float Mn = fmaxf(M[i], mc);
-            const float sa = expf(M[i] - Mn), sb = expf(mc - Mn);  // sa = 0 for the first chunk
-            L[i] = fmaf(L[i], sa, lc * sb);
-            o0[i] = fmaf(o0[i], sa, lo_f(sv[i][j].x) * sb);
-            o1[i] = fmaf(o1[i], sa, lo_f(sv[i][j].y) * sb);
-            M[i] = Mn;
-          }
-    }
-#pragma unroll
-    for (int i = 0; i < 2; ++i)
-      if (has[i]) {
-        const int b = kB == 1 ? 0 : hb[i] / a.H, h = hb[i] - b * a.H;
-        float* dst = vec + (size_t)b * vs + h * a.hd + 2 * q[i];
-        const float inv = 1.0f / L[i];
-        dst[0] = o0[i] * inv;
-        dst[1] = o1[i] * inv;
-      }
   }
   return true;
 }
@@ -869,8 +807,9 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
   const StagePlan* plans = reinterpret_cast<const StagePlan*>(smem + a.sm_misc + kPlansOffset);
   const int tid = threadIdx.x, c = blockIdx.x;
   const int vs = kB == 1 ? 0 : a.vs;
-  // 16-byte polls in flight per thread: one batch covers the 1024 pairs of h
-  // at hidden width 2048
+  // 16-byte polls in flight per thread: one batch covers a 768-wide vector,
+  // and the 1024 pairs of h at hidden width 2048
+  constexpr int kPollDepth = 4;
   constexpr int kPollDepthH = kB == 1 ? 5 : 8;
   const Poll pc{a.err, a.err_host, s_abort, a.wait_limit_ns};
   const unsigned per_step = (unsigned)(kPhasesPerLayer * a.L + 1);
@@ -1004,8 +943,16 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
           else norm_local(gain, ss);
           if (!norm_scales(ok, ss, rs)) return false;
         } else if (k == 1) {
-          // o: the chunk records of every head, merged here
-          if (!vote_ok(merge_records<kB>(a, pos, el + 1, vec, vs, pc), s_abort)) return false;
+          // o, published by the heads' mergers
+          const int hp = a.d >> 1;
+          const bool ok = poll_pairs<kPollDepth>(a.x_attn, kB * hp, el + 1, pc,
+                                                 [&](int p, float v0, float v1) {
+            const int pb = kB == 1 ? 0 : p / hp;
+            float* dst = vec + (size_t)pb * vs + 2 * (p - pb * hp);
+            dst[0] = v0;
+            dst[1] = v1;
+          });
+          if (!vote_ok(ok, s_abort)) return false;
           // Release the K/V rows this CTA wrote in the attention phase: every
           // result it publishes from here on (at the latest its argmax
           // candidate, which every CTA reads before its next step's attention)
