@@ -194,10 +194,7 @@ __global__ void split_bf16_kernel(const float* __restrict__ src, __nv_bfloat16* 
                                   __nv_bfloat16* __restrict__ lo, long long count) {
   for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < count;
        i += (long long)gridDim.x * blockDim.x) {
-    const float v = src[i];
-    const __nv_bfloat16 h = __float2bfloat16_rn(v);
-    hi[i] = h;
-    lo[i] = __float2bfloat16_rn(v - __bfloat162float(h));
+    store_bf16_parts(hi, lo, (size_t)i, src[i]);
   }
 }
 

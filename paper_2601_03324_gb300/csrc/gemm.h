@@ -1,8 +1,20 @@
 // gemm.h — the tensor-core GEMM of gemm.cu for the library's other host files.
 #pragma once
+#include <cuda_bf16.h>
+
 #include "host_common.h"
 
 namespace tvl {
+
+// The bf16 parts of a float32 value v, hi = bf16(v) and lo = bf16(v - hi),
+// stored at index i of hi and lo: the form in which the products below take
+// their operands.
+__device__ __forceinline__ void store_bf16_parts(__nv_bfloat16* hi, __nv_bfloat16* lo, size_t i,
+                                                 float v) {
+  const __nv_bfloat16 h = __float2bfloat16_rn(v);
+  hi[i] = h;
+  lo[i] = __float2bfloat16_rn(v - __bfloat162float(h));
+}
 
 // hi = bf16(src), lo = bf16(src - hi), count floats, on stream s.
 tvl_status split_bf16(const float* src, void* hi, void* lo, long long count, cudaStream_t s);

@@ -23,6 +23,19 @@ namespace {
 
 constexpr int kRowThreads = 256;
 
+// Where a kernel puts rows that a weight product reads next: the bf16 parts
+// (hi, lo) that the tensor-core GEMM takes, written here so that no separate
+// split pass runs; or plain floats (f) when hi is null.
+struct RowOut {
+  float* f;
+  __nv_bfloat16* hi;
+  __nv_bfloat16* lo;
+  __device__ __forceinline__ void put(size_t i, float v) const {
+    if (hi) store_bf16_parts(hi, lo, i, v);
+    else f[i] = v;
+  }
+};
+
 __device__ __forceinline__ float warp_sum32(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -41,10 +54,10 @@ __global__ void embed_rows_kernel(const float* __restrict__ E, const int* __rest
 // then out_{i - row0} = RMSNorm(x_i, g) = (x_i * g) * 1/sqrt(mean x_i^2 + eps)
 // (§11.2); g null: the gain is already in the columns of the next matrix
 // (tvl_load folds it there for float32 rows), so out = x_i * r. Rows
-// [row0, row0 + gridDim.x); out may be add (each row is read in full before it
-// is written).
+// [row0, row0 + gridDim.x); out's floats may be add (each row is read in full
+// before it is written).
 __global__ void rmsnorm_rows_kernel(float* x, const float* add, const float* __restrict__ g,
-                                    float* out, int row0, int d, float eps) {
+                                    RowOut out, int row0, int d, float eps) {
   __shared__ float red[kRowThreads / 32];
   const int i = row0 + blockIdx.x;
   float* xr = x + (size_t)i * d;
@@ -63,8 +76,8 @@ __global__ void rmsnorm_rows_kernel(float* x, const float* add, const float* __r
   float tot = 0.f;
   for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += red[w];
   const float r = 1.0f / sqrtf(tot / (float)d + eps);
-  float* o = out + (size_t)blockIdx.x * d;
-  for (int j = threadIdx.x; j < d; j += blockDim.x) o[j] = (g ? xr[j] * g[j] : xr[j]) * r;
+  const size_t o = (size_t)blockIdx.x * d;
+  for (int j = threadIdx.x; j < d; j += blockDim.x) out.put(o + j, (g ? xr[j] * g[j] : xr[j]) * r);
 }
 
 // RoPE on q and k of row i (position start + i): pair (2m, 2m+1) of a head
@@ -100,7 +113,7 @@ __global__ void rope_kv_kernel(float* __restrict__ qkv, const float2* __restrict
 // of the head (hd <= 128). Four positions per step, their dot products
 // reduced together.
 __global__ void attention_rows_kernel(const float* __restrict__ qkv, const float* __restrict__ kc,
-                                      const float* __restrict__ vc, float* __restrict__ att,
+                                      const float* __restrict__ vc, RowOut att,
                                       int n, int start, int d, int kvd, int hd, int H, int Hkv,
                                       float scale) {
   const int gw = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -158,11 +171,11 @@ __global__ void attention_rows_kernel(const float* __restrict__ qkv, const float
       m = mn;
     }
   }
-  float* out = att + (size_t)i * d + h * hd;
+  const size_t out = (size_t)i * d + h * hd;
 #pragma unroll
   for (int u = 0; u < kMaxPer; ++u) {
     const int j = lane + 32 * u;
-    if (j < hd) out[j] = o[u] / l;
+    if (j < hd) att.put(out + j, o[u] / l);
   }
 }
 
@@ -185,7 +198,7 @@ constexpr int kAttSplits = 8;  // key splits of the longest rows, at most
 template <int kDpt>
 __global__ void __launch_bounds__(kAttThreads)
     attention_tiles_kernel(const float* __restrict__ qkv, const float* __restrict__ kc,
-                           const float* __restrict__ vc, float* __restrict__ att, int n, int start,
+                           const float* __restrict__ vc, RowOut att, int n, int start,
                            int d, int kvd, int H, int Hkv, float scale, int tiles_per_split,
                            float* __restrict__ part) {
   constexpr int hd = 4 * kDpt, hp = hd + 4, hd4 = kDpt, nc = kDpt / 4;
@@ -301,10 +314,15 @@ __global__ void __launch_bounds__(kAttThreads)
       }
     } else {
       const float inv = 1.0f / l;
-      float4* out = reinterpret_cast<float4*>(att + (size_t)(i0 + q) * d + h * hd);
+      const size_t out = (size_t)(i0 + q) * d + h * hd;
 #pragma unroll
-      for (int c = 0; c < nc; ++c)
-        out[4 * c + sub] = make_float4(o[c].x * inv, o[c].y * inv, o[c].z * inv, o[c].w * inv);
+      for (int c = 0; c < nc; ++c) {
+        const size_t e = out + 4 * (4 * c + sub);
+        att.put(e, o[c].x * inv);
+        att.put(e + 1, o[c].y * inv);
+        att.put(e + 2, o[c].z * inv);
+        att.put(e + 3, o[c].w * inv);
+      }
     }
   }
 }
@@ -314,7 +332,7 @@ __global__ void __launch_bounds__(kAttThreads)
 // splits that hold keys of the row's 32-row block (split 0 holds key 0 of every
 // row, so M is finite; a split with no key up to the row has m = -inf and
 // weight 0).
-__global__ void attention_merge_kernel(const float* __restrict__ part, float* __restrict__ att,
+__global__ void attention_merge_kernel(const float* __restrict__ part, RowOut att,
                                        int n, int start, int d, int H, int hd,
                                        int tiles_per_split) {
   const int gw = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -338,12 +356,12 @@ __global__ void attention_merge_kernel(const float* __restrict__ part, float* __
       const float mz = p0[z * stride + hd];
       if (mz != -INFINITY) o = fmaf(expf(mz - M), p0[z * stride + j], o);
     }
-    att[(size_t)i * d + h * hd + j] = o * inv;
+    att.put((size_t)i * d + h * hd + j, o * inv);
   }
 }
 
 template <int kDpt>
-tvl_status launch_attention_tiles(const float* qkv, const float* kc, const float* vc, float* att,
+tvl_status launch_attention_tiles(const float* qkv, const float* kc, const float* vc, RowOut att,
                                   int n, int start, int d, int kvd, int H, int Hkv, float scale,
                                   float* part, cudaStream_t st) {
   constexpr int hp = 4 * kDpt + 4;
@@ -371,12 +389,11 @@ tvl_status launch_attention_tiles(const float* qkv, const float* kc, const float
 
 // h[i][j] = silu(a) * b with (a, b) = rows (2j, 2j + 1) of the interleaved
 // W1/W3 output (§2.1, SwiGLU).
-__global__ void swiglu_rows_kernel(const float* __restrict__ h13, float* __restrict__ h,
-                                   long long total) {
+__global__ void swiglu_rows_kernel(const float* __restrict__ h13, RowOut h, long long total) {
   for (long long t = blockIdx.x * (long long)blockDim.x + threadIdx.x; t < total;
        t += (long long)gridDim.x * blockDim.x) {
     const float a = h13[2 * t], b = h13[2 * t + 1];
-    h[t] = (a / (1.0f + expf(-a))) * b;
+    h.put((size_t)t, (a / (1.0f + expf(-a))) * b);
   }
 }
 
@@ -387,12 +404,10 @@ struct Parts {
   const unsigned char* lo;
 };
 
-// Y[rows x M] = X[rows x K] W^T (everything row-major): X is split into its
-// bf16 parts (xh, xl) first, then the tensor-core GEMM.
-tvl_status gemm_rows(const Parts& w, const float* X, void* xh, void* xl, float* Y, int rows,
-                     int M, int K, int* err, cudaStream_t st) {
-  tvl_status s = split_bf16(X, xh, xl, (long long)rows * K, st);
-  if (s != TVL_OK) return s;
+// Y[rows x M] = X[rows x K] W^T (everything row-major) on the tensor cores,
+// X given as its bf16 parts (xh, xl), which the kernel before wrote.
+tvl_status gemm_rows(const Parts& w, const void* xh, const void* xl, float* Y, int rows, int M,
+                     int K, int* err, cudaStream_t st) {
   return gemm_bf16x3(w.hi, w.lo, xh, xl, Y, rows, M, K, M, err, st);
 }
 
@@ -468,30 +483,30 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
         if (s2 != TVL_OK) return s2;
       }
   }
-  // activations of up to S rows: x, x_b, qkv, att, h13, h; the last row's
-  // normalised vector; the tokens; the bf16 parts of a GEMM input
-  const size_t fx = (size_t)S * d, fqkv = (size_t)S * (d + 2 * kvd), fh13 = (size_t)S * 2 * F,
-               fh = (size_t)S * F;
+  // activations of up to S rows: x, the products' outputs (Wo and W2: y;
+  // [Wq|Wk|Wv]: qkv; W1/W3: h13); the last row's normalised vector; the
+  // tokens; the bf16 parts of the next product's input (the normalised rows,
+  // the attention output or h), written by the kernel that makes them
+  const size_t fx = (size_t)S * d, fqkv = (size_t)S * (d + 2 * kvd), fh13 = (size_t)S * 2 * F;
   const size_t xpart = al(2ull * S * (d > F ? d : F));
   // partials (o, max, sum) of the attention's key splits
   const size_t fpart = (size_t)kAttSplits * S * a.H * (hd + 4);
-  const size_t need = al(4 * (3 * fx + fqkv + fh13 + fh + d) + 4 * (size_t)S) + 2 * xpart +
-                      al(4 * fpart);
+  const size_t fbytes = al(4 * (2 * fx + fqkv + fh13 + d) + 4 * (size_t)S);
+  const size_t need = fbytes + 2 * xpart + al(4 * fpart);
   if (!m->pf) {
     TVL_CK(lib_malloc((void**)&m->pf, need));
     m->pf_bytes = need;
   }
   float* X = m->pf;
-  float* XB = X + fx;
-  float* QKV = XB + fx;
-  float* ATT = QKV + fqkv;
-  float* H13 = ATT + fx;
-  float* Hh = H13 + fh13;
-  float* XN = Hh + fh;
+  float* Y = X + fx;
+  float* QKV = Y + fx;
+  float* H13 = QKV + fqkv;
+  float* XN = H13 + fh13;
   int* tok = reinterpret_cast<int*>(XN + d);
-  unsigned char* xh = reinterpret_cast<unsigned char*>(m->pf) +
-                      al(4 * (3 * fx + fqkv + fh13 + fh + d) + 4 * (size_t)S);
+  unsigned char* xh = reinterpret_cast<unsigned char*>(m->pf) + fbytes;
   unsigned char* xl = xh + xpart;
+  const RowOut parts{nullptr, reinterpret_cast<__nv_bfloat16*>(xh),
+                     reinterpret_cast<__nv_bfloat16*>(xl)};
   float* PART = reinterpret_cast<float*>(xl + xpart);
   int* err = nullptr;
   tvl_status s = gemm_error_word(&err);
@@ -507,9 +522,9 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
     const float* g_ffn = a.gains_folded ? nullptr : reinterpret_cast<const float*>(lw + a.o_gffn);
     float* kc = a.kc + (size_t)l * S * kvd;
     float* vc = a.vc + (size_t)l * S * kvd;
-    rmsnorm_rows_kernel<<<n, kRowThreads, 0, st>>>(X, pending, g_att, XB, 0, d, a.eps);
+    rmsnorm_rows_kernel<<<n, kRowThreads, 0, st>>>(X, pending, g_att, parts, 0, d, a.eps);
     TVL_CK(cudaGetLastError());
-    if ((s = gemm_rows(wparts(l, 0), XB, xh, xl, QKV, n, d + 2 * kvd, d, err, st)) != TVL_OK)
+    if ((s = gemm_rows(wparts(l, 0), xh, xl, QKV, n, d + 2 * kvd, d, err, st)) != TVL_OK)
       return s;
     rope_kv_kernel<<<n, kRowThreads, 0, st>>>(QKV, a.rope, kc, vc, start_pos, d, kvd, hd);
     TVL_CK(cudaGetLastError());
@@ -517,39 +532,39 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
       const float sc = a.att_scale;
       s = TVL_OK;
       switch (hd) {
-        case 16: s = launch_attention_tiles<4>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
-        case 32: s = launch_attention_tiles<8>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
-        case 48: s = launch_attention_tiles<12>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
-        case 64: s = launch_attention_tiles<16>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
-        case 80: s = launch_attention_tiles<20>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
-        case 96: s = launch_attention_tiles<24>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
-        case 112: s = launch_attention_tiles<28>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
-        case 128: s = launch_attention_tiles<32>(QKV, kc, vc, ATT, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 16: s = launch_attention_tiles<4>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 32: s = launch_attention_tiles<8>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 48: s = launch_attention_tiles<12>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 64: s = launch_attention_tiles<16>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 80: s = launch_attention_tiles<20>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 96: s = launch_attention_tiles<24>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 112: s = launch_attention_tiles<28>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 128: s = launch_attention_tiles<32>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
         default: {
           const int warps = n * a.H, wpb = kRowThreads / 32;
           attention_rows_kernel<<<(warps + wpb - 1) / wpb, kRowThreads, 0, st>>>(
-              QKV, kc, vc, ATT, n, start_pos, d, kvd, hd, a.H, a.Hkv, a.att_scale);
+              QKV, kc, vc, parts, n, start_pos, d, kvd, hd, a.H, a.Hkv, a.att_scale);
           TVL_CK(cudaGetLastError());
         }
       }
       if (s != TVL_OK) return s;
     }
-    // XB = Wo o
-    if ((s = gemm_rows(wparts(l, 1), ATT, xh, xl, XB, n, d, d, err, st)) != TVL_OK) return s;
-    rmsnorm_rows_kernel<<<n, kRowThreads, 0, st>>>(X, XB, g_ffn, ATT, 0, d, a.eps);  // ATT = x_b
+    // Y = Wo o; x += Y and the parts of x_b = RMSNorm(x)
+    if ((s = gemm_rows(wparts(l, 1), xh, xl, Y, n, d, d, err, st)) != TVL_OK) return s;
+    rmsnorm_rows_kernel<<<n, kRowThreads, 0, st>>>(X, Y, g_ffn, parts, 0, d, a.eps);
     TVL_CK(cudaGetLastError());
-    if ((s = gemm_rows(wparts(l, 2), ATT, xh, xl, H13, n, 2 * F, d, err, st)) != TVL_OK) return s;
+    if ((s = gemm_rows(wparts(l, 2), xh, xl, H13, n, 2 * F, d, err, st)) != TVL_OK) return s;
     const long long tot = (long long)n * F;
-    swiglu_rows_kernel<<<(int)std::min<long long>((tot + 255) / 256, 4096), 256, 0, st>>>(H13, Hh,
+    swiglu_rows_kernel<<<(int)std::min<long long>((tot + 255) / 256, 4096), 256, 0, st>>>(H13, parts,
                                                                                         tot);
     TVL_CK(cudaGetLastError());
-    // XB = W2 h
-    if ((s = gemm_rows(wparts(l, 3), Hh, xh, xl, XB, n, d, F, err, st)) != TVL_OK) return s;
-    pending = XB;
+    // Y = W2 h
+    if ((s = gemm_rows(wparts(l, 3), xh, xl, Y, n, d, F, err, st)) != TVL_OK) return s;
+    pending = Y;
   }
   // the last position: x += (last update), x_b = RMSNorm(x, g_final), logits = Wcls x_b
   rmsnorm_rows_kernel<<<1, kRowThreads, 0, st>>>(X, pending, a.final_gain_folded ? nullptr : a.g_final,
-                                                  XN, n - 1, d, a.eps);
+                                                  RowOut{XN, nullptr, nullptr}, n - 1, d, a.eps);
   TVL_CK(cudaGetLastError());
   if ((s = tvl_gemv(a.Wcls, XN, a.logits, V, d, st)) != TVL_OK) return s;
   if (!logits_out) return TVL_OK;
