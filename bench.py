@@ -60,8 +60,7 @@ def parse():
     ap.add_argument("--impl", default="tvl", choices=["tvl", "reference"])
     ap.add_argument("--workload", default="110m", choices=["110m", "110m-long", "tiny", "7b"])
     ap.add_argument("--weights", default="f32", choices=["f32", "q8", "q4"],
-                    help="q8: weight-only 8-bit rows (tvl_config.weight_bits = 8); "
-                         "q4: weight-only 4-bit rows (--gemv-sweep only)")
+                    help="q8 / q4: weight-only 8-bit / 4-bit rows (tvl_config.weight_bits)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
@@ -263,15 +262,20 @@ def cpu_decode_rate(make, cfg, seconds: float):
     return n / el, n, el
 
 
+WEIGHT_BITS = {"f32": 0, "q8": 8, "q4": 4}  # tvl_config.weight_bits of each --weights
+
+
 def streamed_bytes_of(cfg: dict, weight_bits: int = 0) -> int:
     """Weight bytes one decode step reads: every matrix and gain of every
     layer, one embedding row, the final gain and the classifier (8-bit rows:
-    16 + K bytes per row)."""
+    16 + K bytes per row; 4-bit rows: 16 + K / 2)."""
     d, F, L, V = cfg["dim"], cfg["hidden_dim"], cfg["n_layers"], cfg["vocab_size"]
     kvd = cfg["n_kv_heads"] * (d // cfg["n_heads"])
-    if weight_bits == 8:
-        return (L * ((d + 2 * kvd) * (16 + d) + d * (16 + d) + 2 * F * (16 + d) + d * (16 + F)
-                     + 8 * d) + V * (16 + d) + (16 + d) + 4 * d)
+    if weight_bits in (8, 4):
+        rq = 16 + (d if weight_bits == 8 else d // 2)
+        rf = 16 + (F if weight_bits == 8 else F // 2)
+        return (L * ((d + 2 * kvd) * rq + d * rq + 2 * F * rq + d * rf + 8 * d) + V * rq + rq
+                + 4 * d)
     return 4 * (L * ((d + 2 * kvd) * d + d * d + 3 * F * d + 2 * d) + V * d + 2 * d)
 
 
@@ -515,10 +519,6 @@ def prefill_bench(args, cfg):
 
 def main():
     args = parse()
-    if args.weights == "q4" and not args.gemv_sweep:
-        print(json.dumps({"error": "--weights q4 is for --gemv-sweep: models decode with "
-                                   "float32 or 8-bit rows"}))
-        return 2
     rank, local_rank, world = dist_env()
     from paper_2601_03324_gb300 import synth
     cfg = synth.model_config("110m" if args.workload == "110m-long" else args.workload)
@@ -541,8 +541,8 @@ def main():
                                    "110m-long"}))
         return 2
     blob = synth.make_blob(cfg)
-    if args.weights == "q8":
-        cfg = dict(cfg, weight_bits=8)
+    if args.weights in ("q8", "q4"):
+        cfg = dict(cfg, weight_bits=WEIGHT_BITS[args.weights])
     if B > 1:
         cfg = dict(cfg, max_batch=B)
     stream = torch.cuda.Stream()
@@ -634,7 +634,7 @@ def main():
     bytes_launch = bytes_timed / len(per)
     peak, peak_src = measured_peaks()
     achieved = bytes_timed / (kern_ms * 1e-3) / 1e9
-    traffic = committed_traffic(args.workload + ("_q8" if args.weights == "q8" else "") +
+    traffic = committed_traffic(args.workload + ("" if args.weights == "f32" else "_" + args.weights) +
                                 (f"_b{B}" if B > 1 else ""), bytes_launch)
 
     # one whole sequence on its own (not part of the timed region)
@@ -715,7 +715,7 @@ def main():
     cpu = cpu_pm = None
     if rank == 0 and not args.no_cpu_baseline and args.workload in ("110m", "tiny"):
         import oracle
-        wb = 8 if args.weights == "q8" else 0
+        wb = WEIGHT_BITS[args.weights]
         rate, n, el = cpu_decode_rate(lambda: oracle.Model(cfg, blob, 32, weight_bits=wb), cfg,
                                       args.cpu_seconds)
         cpu = {"value": rate, "unit": "tokens/s", "cores": 1, "kind": "oracle",
@@ -740,7 +740,7 @@ def main():
         energy = {"power_w": clk["power_w"],
                   "mj_per_token": 1e3 * clk["power_w"] * (el_ms * 1e-3) / (args.steps * B),
                   "note": "nvidia-smi power.draw (board), median over the timed region"}
-    streamed_cfg = streamed_bytes_of(cfg, 8 if args.weights == "q8" else 0)
+    streamed_cfg = streamed_bytes_of(cfg, WEIGHT_BITS[args.weights])
     assert streamed_cfg == info.streamed_bytes, (streamed_cfg, info.streamed_bytes)
     line = {
         "metric": METRIC if B == 1 else METRIC_BATCH.format(b=B), "value": value,
@@ -749,7 +749,8 @@ def main():
         "higher_is_better": True, "scaling": "weak",
         "vs_baseline": (value / PAPER_TOKS
                         if args.workload == "110m" and args.weights == "f32" and B == 1 else None),
-        "dtype": "f32" if args.weights == "f32" else "f32 activations, int8 weight rows",
+        "dtype": {"f32": "f32", "q8": "f32 activations, int8 weight rows",
+                  "q4": "f32 activations, int4 weight rows"}[args.weights],
         "data": "synthetic (seeded N(0, 0.02) weights)",
         "config": workload_config(args.workload, cfg, B, args.weights, positions_of(wins)),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",

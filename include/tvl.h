@@ -53,8 +53,9 @@ typedef struct {
   int32_t weight_bits;  /* 0: float32 weights as in the blob; 8: tvl_load turns every weight
                            matrix (and the embedding table) into 8-bit rows, as
                            tvl_quantize_q8 defines, and decodes with them; dim and
-                           hidden_dim must then be multiples of 16. Any other value is
-                           TVL_E_INVAL (4-bit rows serve the standalone tvl_gemv_q4 only) */
+                           hidden_dim must then be multiples of 16; 4: the same with
+                           4-bit rows as tvl_quantize_q4 defines (dim and hidden_dim
+                           multiples of 32). Any other value is TVL_E_INVAL */
   int32_t max_batch;    /* sequences one launch may decode together, 0 or 1 (one) to 4;
                            each sequence slot gets its own KV cache and exchange buffers.
                            More than one needs weight_bits 0 */
@@ -156,7 +157,7 @@ tvl_status tvl_decode_greedy_batch(tvl_model* m, int32_t batch, const int32_t* s
  *   logits_out: V floats, as for tvl_forward (device: no wait; host: waits;
  *   NULL: kept on the device).
  *   n >= 1, start_pos >= 0, start_pos + n <= max_seq, tokens in [0, V), else
- *   TVL_E_RANGE; a model loaded with weight_bits 8: TVL_E_UNSUPPORTED. */
+ *   TVL_E_RANGE; a model loaded with weight_bits 8 or 4: TVL_E_UNSUPPORTED. */
 tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n, int32_t start_pos,
                        float* logits_out);
 
@@ -239,7 +240,7 @@ tvl_status tvl_quantize_q4(const float* W, void* Wq4, int32_t rows, int32_t cols
  * sum_j q[r][j] x[j]); Wq4 and x device pointers, 16-byte aligned; d_in a
  * multiple of 32 and at most 32736 (a packed row fits one 16 KB stage), else
  * TVL_E_INVAL / TVL_E_ALIGN / TVL_E_UNSUPPORTED. Queued on `stream`, does not
- * wait, allocates nothing. Models decode with float32 or 8-bit rows only. */
+ * wait, allocates nothing. */
 tvl_status tvl_gemv_q4(const void* Wq4, const float* x, float* y, int32_t d_out, int32_t d_in,
                        void* stream);
 

@@ -69,7 +69,7 @@ bool config_valid(const tvl_config* c) {
   if ((c->dim / c->n_heads) % 2 != 0) return false;  // RoPE turns pairs
   if (!(c->rope_theta > 0.0) || !(c->norm_eps >= 0.0)) return false;
   if (c->shared_classifier < -1 || c->shared_classifier > 1) return false;
-  if (c->weight_bits != 0 && c->weight_bits != 8) return false;
+  if (c->weight_bits != 0 && c->weight_bits != 8 && c->weight_bits != 4) return false;
   if (c->max_batch < 0 || c->max_batch > 4) return false;
   return true;
 }

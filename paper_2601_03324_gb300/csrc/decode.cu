@@ -211,7 +211,8 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
               "hidden_dim % 4 == 0, max(dim, hidden_dim) <= 16384");
     return TVL_E_UNSUPPORTED;
   }
-  const bool q8 = cfg->weight_bits == 8;
+  const bool q4 = cfg->weight_bits == 4;
+  const bool q8 = cfg->weight_bits == 8 || q4;  // quantized rows, 8-bit or 4-bit
   const int maxB = cfg->max_batch > 1 ? cfg->max_batch : 1;
   if (maxB > 1 && q8) {
     set_error("tvl_load: max_batch > 1 needs float32 weights (weight_bits 0)");
@@ -219,6 +220,10 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   }
   if (q8 && (d % 16 != 0 || F % 16 != 0 || std::max(d, F) > 16368)) {
     set_error("tvl_load: 8-bit rows need dim and hidden_dim multiples of 16 and at most 16368");
+    return TVL_E_UNSUPPORTED;
+  }
+  if (q4 && (d % 32 != 0 || F % 32 != 0)) {
+    set_error("tvl_load: 4-bit rows need dim and hidden_dim multiples of 32");
     return TVL_E_UNSUPPORTED;
   }
   // §5.1 weight tying: explicit, or inferred from the blob size.
@@ -254,7 +259,9 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
     return e == cudaSuccess ? TVL_OK : cuda_fail(e, what);
   };
   tvl_status st;
-  m->kernel[1] = q8 ? (const void*)decode_kernel<true, 1> : (const void*)decode_kernel<false, 1>;
+  m->kernel[1] = q4   ? (const void*)decode_kernel<true, 1, true>
+                 : q8 ? (const void*)decode_kernel<true, 1>
+                      : (const void*)decode_kernel<false, 1>;
   for (int B = 2; B <= maxB; ++B) m->kernel[B] = decode_kernel_for_batch(B);
   if ((st = ck(cudaGetDevice(&m->device), "cudaGetDevice")) != TVL_OK) return fail(st);
   int sms = 0, coop = 0, max_optin = 0;
@@ -315,8 +322,8 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
     return at;
   };
   const size_t o_w = take(blob_bytes);
-  // 8-bit rows: per layer [Wq|Wk|Wv], Wo, [W1|W3], W2; then E and the untied classifier
-  const size_t rq = 16 + (size_t)d, rf = 16 + (size_t)F;
+  // quantized rows: per layer [Wq|Wk|Wv], Wo, [W1|W3], W2; then E and the untied classifier
+  const size_t rq = 16 + (size_t)(q4 ? d / 2 : d), rf = 16 + (size_t)(q4 ? F / 2 : F);
   size_t q_wqkv = 0, q_wo = 0, q_w13 = 0, q_w2 = 0, q_stride = 0, o_q = 0, o_qE = 0, o_qcls = 0;
   if (q8) {
     size_t lo = 0;
@@ -397,11 +404,13 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   if (st == TVL_OK) st = ck(cudaStreamSynchronize(m->stream), "cudaStreamSynchronize(blob)");
   if (registered) cudaHostUnregister(const_cast<void*>(blob));
   if (st != TVL_OK) return fail(st);
-  if (q8) {  // every weight matrix to 8-bit rows, on the device (tvl_quantize_q8)
+  if (q8) {  // every weight matrix to 8-bit (or 4-bit) rows, on the device
     const unsigned char* Wf = m->arena + o_w;
     auto quant = [&](const unsigned char* src, size_t dst, int rows, int cols) {
-      return tvl_quantize_q8(reinterpret_cast<const float*>(src), m->arena + dst, rows, cols,
-                             m->stream);
+      return q4 ? tvl_quantize_q4(reinterpret_cast<const float*>(src), m->arena + dst, rows, cols,
+                                  m->stream)
+                : tvl_quantize_q8(reinterpret_cast<const float*>(src), m->arena + dst, rows, cols,
+                                  m->stream);
     };
     for (int l = 0; l < L && st == TVL_OK; ++l) {
       const unsigned char* lw = Wf + bl.l0 + (size_t)l * bl.stride;
@@ -516,9 +525,9 @@ tvl_status tvl_load(const tvl_config* cfg, const void* blob, size_t blob_bytes, 
   a.kv_seq = (long long)kv_seq;
   a.wait_limit_ns = kWaitLimitNs;
   m->streamed_bytes =
-      q8 ? (int64_t)L * ((int64_t)(d + 2 * kvd) * (16 + d) + (int64_t)d * (16 + d) +
-                         2LL * F * (16 + d) + (int64_t)d * (16 + F) + 8LL * d) +
-               (int64_t)V * (16 + d) + (16 + d) + 4LL * d
+      q8 ? (int64_t)L * ((int64_t)(d + 2 * kvd) * (int64_t)rq + (int64_t)d * (int64_t)rq +
+                         2LL * F * (int64_t)rq + (int64_t)d * (int64_t)rf + 8LL * d) +
+               (int64_t)V * (int64_t)rq + (int64_t)rq + 4LL * d
          : 4LL * ((int64_t)L * ((int64_t)(d + 2 * kvd) * d + (int64_t)d * d + 3LL * F * d + 2LL * d) +
                   (int64_t)V * d + 2LL * d);
   *out = m;

@@ -745,10 +745,12 @@ static_assert(kPlansOffset + 5 * sizeof(StagePlan) <= kMiscBytes, "stage plans o
 
 // This CTA's stage plans of the five GEMV kinds — [Wq|Wk|Wv], Wo, W1/W3
 // (interleaved row pairs), W2, the classifier — the same in every layer and
-// step, so they are worked out once per launch (8-bit rows are 4 + K/4 words).
-template <bool kQ8>
+// step, so they are worked out once per launch (8-bit rows are 4 + K/4 words,
+// 4-bit rows 4 + K/8).
+template <bool kQ8, bool kQ4 = false>
 __device__ inline void phase_plans(const DecodeArgs& a, int c, StagePlan* plans) {
-  const int kd = kQ8 ? 4 + a.d / 4 : a.d, kf = kQ8 ? 4 + a.F / 4 : a.F;
+  const int kd = kQ4 ? 4 + a.d / 8 : kQ8 ? 4 + a.d / 4 : a.d;
+  const int kf = kQ4 ? 4 + a.F / 8 : kQ8 ? 4 + a.F / 4 : a.F;
   plans[0] = plan_stages(a.d + 2 * a.kvd, kd, a.G, c);
   plans[1] = plan_stages(a.d, kd, a.G, c);
   plans[2] = plan_stages(2 * a.F, kd, a.G, c, 2);
@@ -795,7 +797,8 @@ struct DecodeSched {
 // kB sequences decode in lockstep: sequence b's residual at xs + b d, its
 // phase input at vec + b vs, its words in every exchange buffer one vector
 // length after sequence b - 1's. The weights stream once for all of them.
-template <bool kQ8, int kB>
+// kQ8: quantized rows (8-bit, or 4-bit with kQ4).
+template <bool kQ8, int kB, bool kQ4 = false>
 __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned char* smem,
                                     volatile int* s_abort) {
   float* xs = reinterpret_cast<float*>(smem + a.sm_xs);
@@ -895,7 +898,22 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
 #pragma unroll
     for (int b = 0; b < kB; ++b) {
       float* xb = xs + (size_t)b * a.d;
-      if (kQ8) {  // the row the codes stand for: scale * code
+      if (kQ4) {  // the row the 4-bit codes stand for: scale * code
+        const unsigned char* er = a.q_E + (size_t)token[b] * (16 + a.d / 2);
+        const float sc = __ldg(reinterpret_cast<const float*>(er));
+        const unsigned* cw = reinterpret_cast<const unsigned*>(er + 16);
+        for (int j = tid; j < (a.d >> 3); j += kConsumerThreads) {
+          const unsigned w = __ldg(cw + j);
+          float v[8];
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const int c4 = (int)((w >> (4 * k)) & 0xFu);
+            v[k] = sc * (float)(c4 >= 8 ? c4 - 16 : c4);
+          }
+          reinterpret_cast<float4*>(xb)[2 * j] = make_float4(v[0], v[1], v[2], v[3]);
+          reinterpret_cast<float4*>(xb)[2 * j + 1] = make_float4(v[4], v[5], v[6], v[7]);
+        }
+      } else if (kQ8) {  // the row the codes stand for: scale * code
         const unsigned char* er = a.q_E + (size_t)token[b] * (16 + a.d);
         const float sc = __ldg(reinterpret_cast<const float*>(er));
         const int* cw = reinterpret_cast<const int*>(er + 16);
@@ -980,8 +998,8 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
                  {rs[0], rs[1], rs[2], rs[3]}};
         if constexpr (kQ8) {
           uint32_t g = cur.g;
-          if (!consume_phase<false, kQ8>(r, g, plan, vec, 1, K, seg, e, a.err, a.err_host,
-                                         s_abort))
+          if (!consume_phase<false, kQ8, kQ4>(r, g, plan, vec, 1, K, seg, e, a.err, a.err_host,
+                                              s_abort))
             return false;
           cur.advance(plan.nstages, r.nst);
         } else {
@@ -1005,8 +1023,8 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
     ea.init();
     if constexpr (kQ8) {
       uint32_t g = cur.g;
-      if (!consume_phase<false, kQ8>(r, g, plans[4], vec, 1, a.d, seg, ea, a.err, a.err_host,
-                                     s_abort))
+      if (!consume_phase<false, kQ8, kQ4>(r, g, plans[4], vec, 1, a.d, seg, ea, a.err,
+                                          a.err_host, s_abort))
         return false;
       cur.advance(plans[4].nstages, r.nst);
     } else {
@@ -1039,7 +1057,7 @@ __device__ inline bool decode_steps(const DecodeArgs& a, const Ring& r, unsigned
   return true;
 }
 
-template <bool kQ8, int kB>
+template <bool kQ8, int kB, bool kQ4 = false>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_constant__ DecodeArgs a) {
   extern __shared__ __align__(128) unsigned char smem[];
   Ring r;
@@ -1056,7 +1074,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
       r.seq[i] = 0;
     }
     *s_abort = 0;
-    phase_plans<kQ8>(a, blockIdx.x, reinterpret_cast<StagePlan*>(smem + a.sm_misc + kPlansOffset));
+    phase_plans<kQ8, kQ4>(a, blockIdx.x,
+                          reinterpret_cast<StagePlan*>(smem + a.sm_misc + kPlansOffset));
     fence_mbar_init();
   }
   __syncthreads();
@@ -1069,7 +1088,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
     }
     return;
   }
-  decode_steps<kQ8, kB>(a, r, smem, s_abort);
+  decode_steps<kQ8, kB, kQ4>(a, r, smem, s_abort);
 }
 
 // decode_kernel<false, B> for B = 2..kMaxBatch (defined in decode_batch.cu).

@@ -385,18 +385,21 @@ __device__ __forceinline__ void fma_nibbles(float4& acc, int w, const float4& xa
                                             const float4& xb) {
   // code + 8 (in [1, 15]) as the low bits of the float 2^23 + (code + 8):
   // a shift, a mask and an OR per code, then one exact subtraction
+  // even columns (low nibbles) and odd columns (high nibbles) as bytes, then
+  // each byte into the float 2^23 + (code + 8) by one byte permute
   const unsigned u = (unsigned)w ^ 0x88888888u;
-  auto c = [u](int k) {
-    return __uint_as_float(0x4B000000u | ((u >> (4 * k)) & 0xFu)) - 8388616.0f;
+  const unsigned ev = u & 0x0F0F0F0Fu, od = (u >> 4) & 0x0F0F0F0Fu;
+  auto c = [](unsigned v, unsigned sel) {
+    return __uint_as_float(__byte_perm(v, 0x4B000000u, sel)) - 8388616.0f;
   };
-  acc.x = fmaf(c(0), xa.x, acc.x);
-  acc.y = fmaf(c(1), xa.y, acc.y);
-  acc.z = fmaf(c(2), xa.z, acc.z);
-  acc.w = fmaf(c(3), xa.w, acc.w);
-  acc.x = fmaf(c(4), xb.x, acc.x);
-  acc.y = fmaf(c(5), xb.y, acc.y);
-  acc.z = fmaf(c(6), xb.z, acc.z);
-  acc.w = fmaf(c(7), xb.w, acc.w);
+  acc.x = fmaf(c(ev, 0x7540), xa.x, acc.x);  // column 0
+  acc.y = fmaf(c(od, 0x7540), xa.y, acc.y);  // column 1
+  acc.z = fmaf(c(ev, 0x7541), xa.z, acc.z);  // column 2
+  acc.w = fmaf(c(od, 0x7541), xa.w, acc.w);  // column 3
+  acc.x = fmaf(c(ev, 0x7542), xb.x, acc.x);  // column 4
+  acc.y = fmaf(c(od, 0x7542), xb.y, acc.y);  // column 5
+  acc.z = fmaf(c(ev, 0x7543), xb.z, acc.z);  // column 6
+  acc.w = fmaf(c(od, 0x7543), xb.w, acc.w);  // column 7
 }
 
 // Lane partials of sum_j q_j x_j for two 4-bit rows sharing x (nw code words).

@@ -96,3 +96,52 @@ def test_q4_rejects_bad_shapes(tvl):
         tvl.tvl_quantize_q4(d.data_ptr(), d.data_ptr(), 4, 16)
     with pytest.raises(tvl.TvlError):
         tvl.tvl_gemv_q4(d.data_ptr(), d.data_ptr(), d.data_ptr(), 1, 32768)  # row over a stage
+
+
+# ---- decode with 4-bit weight rows (tvl_config.weight_bits = 4) vs the oracle's
+# model over the same codes; tolerances as for the float32 decode ----
+
+from helpers import compare_greedy, lockstep_greedy, small_config  # noqa: E402
+
+
+def check_q4_model(tvl, cfg, blob, n_steps, start=1, check_every=1, label=""):
+    cfg = dict(cfg, weight_bits=4)
+    ref = oracle.Model(cfg, blob, 64, weight_bits=4)
+    with tvl.Model(cfg, blob) as m:
+        toks, ref_logits, worst = lockstep_greedy(m, ref, start, n_steps,
+                                                  check_every=check_every, label=label)
+        gen = m.decode_greedy(start, 0, n_steps)
+        compare_greedy(gen, toks[1:] + [int(np.argmax(ref_logits[-1]))], ref_logits)
+    return worst
+
+
+def test_q4_tiny_model_64_steps(tvl):
+    cfg = synth.model_config("tiny")
+    check_q4_model(tvl, cfg, synth.make_blob(cfg), cfg["steps"], label="tiny q4")
+
+
+@pytest.mark.parametrize("kw", [
+    dict(),
+    dict(n_kv_heads=2),
+    dict(n_layers=0, shared_classifier=1),
+    dict(dim=128, n_heads=1, n_kv_heads=1, hidden_dim=256, shared_classifier=1),
+], ids=["base", "gqa2", "L0_tied", "hd128_tied"])
+def test_q4_small_shapes_match_oracle(tvl, kw):
+    cfg = small_config(**kw)
+    check_q4_model(tvl, cfg, synth.make_blob(cfg, seed=29), cfg["max_seq"], label=f"q4 {kw}")
+
+
+def test_q4_110m_64_steps(tvl):
+    cfg = synth.model_config("110m")
+    check_q4_model(tvl, cfg, synth.make_blob(cfg), 64, check_every=8, label="110m q4")
+
+
+def test_q4_streams_an_eighth_of_the_float_bytes(tvl):
+    cfg = synth.model_config("110m")
+    blob = synth.make_blob(cfg)
+    with tvl.Model(cfg, blob) as mf, tvl.Model(dict(cfg, weight_bits=4), blob) as mq:
+        sf, sq = mf.info().streamed_bytes, mq.info().streamed_bytes
+    d, F, L, V = cfg["dim"], cfg["hidden_dim"], cfg["n_layers"], cfg["vocab_size"]
+    rq, rf = 16 + d // 2, 16 + F // 2
+    expect = L * ((3 * d) * rq + d * rq + 2 * F * rq + d * rf + 8 * d) + V * rq + rq + 4 * d
+    assert sq == expect and 0.12 < sq / sf < 0.14
