@@ -52,6 +52,33 @@ def test_decode_across_the_exchange_tag_wrap(tvl):
         assert m.info().next_tag == 1 + 14 * per_step
 
 
+def test_lowering_the_next_tag_clears_the_exchange_words(tvl):
+    # Words are published as the unsigned maximum of the old and the new word,
+    # so a tag below those the words hold would never show: lowering the tag
+    # must zero the words first. Decode, go back to tag 1, decode on (the
+    # teacher-forced logits and a greedy launch), parity throughout.
+    cfg = small_config(n_layers=2)
+    blob = synth.make_blob(cfg, seed=22)
+    ref = oracle.Model(cfg, blob)
+    toks, logits = ref.greedy(1, 20)
+    per_step = 5 * cfg["n_layers"] + 1
+    with tvl.Model(cfg, blob) as m:
+        out = np.empty(cfg["vocab_size"], np.float32)
+        for p in range(5):
+            m.forward(toks[p], p, out)
+            assert_logits_close(out, logits[p], f"pos {p}")
+        assert m.info().next_tag == 1 + 5 * per_step
+        tvl._check(tvl.lib.tvl_debug_set_next_tag(m._h, 1), "tvl_debug_set_next_tag")
+        assert m.info().next_tag == 1
+        for p in range(5, 8):
+            m.forward(toks[p], p, out)
+            assert_logits_close(out, logits[p], f"after lowering the tag, pos {p}")
+        tvl._check(tvl.lib.tvl_debug_set_next_tag(m._h, 2), "tvl_debug_set_next_tag")
+        gen = m.decode_greedy(toks[8], 8, 11)  # positions 8..18: oracle tokens 9..19
+        compare_greedy(gen, toks[9:], logits[8:])
+        assert m.info().next_tag == 2 + 11 * per_step
+
+
 def test_set_next_tag_rejects_zero_and_values_beyond_32_bits(tvl):
     cfg = small_config(n_layers=1)
     with tvl.Model(cfg, synth.make_blob(cfg, seed=2)) as m:
