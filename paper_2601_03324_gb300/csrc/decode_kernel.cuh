@@ -696,16 +696,17 @@ __device__ inline bool attention_phase(const DecodeArgs& a, int l, int pos, unsi
             rr[k == 0 ? 1 : 2 * k + 1] = x1;
           });
       if (!vote_ok(ok2, pc.s_abort)) return false;
-      if (tid < hd) {
+      if (tid < hd) {  // one exponential per chunk, one division
         float M = m;
         for (int cc = 0; cc < nch - 1; ++cc) M = fmaxf(M, mrg[cc * (hd + 2)]);
-        float Lsum = expf(m - M) * ls;
-        for (int cc = 0; cc < nch - 1; ++cc)
-          Lsum += expf(mrg[cc * (hd + 2)] - M) * mrg[cc * (hd + 2) + 1];
-        float o = (expf(m - M) / Lsum) * own;
-        for (int cc = 0; cc < nch - 1; ++cc)
-          o = fmaf(expf(mrg[cc * (hd + 2)] - M) / Lsum, mrg[cc * (hd + 2) + 2 + tid], o);
-        st_tag(a.x_attn + (size_t)hb * hd + tid, tag_att, o);
+        const float e0 = expf(m - M);
+        float Lsum = e0 * ls, o = e0 * own;
+        for (int cc = 0; cc < nch - 1; ++cc) {
+          const float e = expf(mrg[cc * (hd + 2)] - M);
+          Lsum = fmaf(e, mrg[cc * (hd + 2) + 1], Lsum);
+          o = fmaf(e, mrg[cc * (hd + 2) + 2 + tid], o);
+        }
+        st_tag(a.x_attn + (size_t)hb * hd + tid, tag_att, o / Lsum);
       }
     }
     named_bar_sync(kBarConsumers, kConsumerThreads);
