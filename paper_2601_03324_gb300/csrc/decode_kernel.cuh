@@ -17,7 +17,8 @@
 // CTA's shared memory: each CTA adds the same values in the same order.
 //
 // Exchange between phases: every value a phase publishes is one 64-bit word,
-// (epoch tag << 32) | float bits, stored once. A reader polls the words it
+// (epoch tag << 32) | float bits, written once (an unsigned-max reduction:
+// tags only grow, so the new word wins). A reader polls the words it
 // needs until each carries the epoch of the current (step, layer, phase); the
 // wait and the read are the same L2 round trip, and no grid-wide barrier is
 // needed. A buffer is rewritten only one layer later, after an exchange that
