@@ -64,6 +64,7 @@ def test_blob_bytes_agree_with_generator_and_oracle(tvl):
     (dict(max_batch=5), "E_INVAL"),                             # 0 to 4 sequences
     (dict(max_batch=-1), "E_INVAL"),
     (dict(max_batch=2, weight_bits=8), "E_UNSUPPORTED"),        # batches need float32 rows
+    (dict(max_batch=3, weight_bits=4), "E_UNSUPPORTED"),
 ])
 def test_load_rejects_invalid_configs_on_the_host(tvl, bad, status):
     cfg = dict(dim=64, hidden_dim=96, n_layers=1, n_heads=4, n_kv_heads=4, vocab_size=100,
