@@ -327,6 +327,175 @@ __global__ void __launch_bounds__(kAttThreads)
   }
 }
 
+// The same causal attention with more work per thread, for head dims that
+// are multiples of 32 (kDpt = head_dim / 4 a multiple of 8): a CTA of 128
+// threads takes 64 query rows of one head and walks its share of the keys in
+// tiles of 32. The tile kernel above reads about one shared-memory value per
+// multiply-add and is bound by the shared-memory port; here each thread keeps
+// a 4 x 4 block of scores (queries 4g .. 4g + 3 of its group g = tid / 8,
+// keys j, j + 8, j + 16, j + 24 of the tile for j = tid % 8) and a 4-query
+// block of the output (float4 chunks j, j + 8, ... of the head's dims), so
+// every value read from shared memory meets four others. The eight threads of
+// a group are lanes of one warp: the scores' row maxima and sums are shuffles
+// among them, and the softmax weights go through shared memory within the
+// warp. Key splits and partials as above.
+constexpr int kAtt2BQ = 64;
+
+template <int kDpt>
+__global__ void __launch_bounds__(kAttThreads)
+    attention_tiles64_kernel(const float* __restrict__ qkv, const float* __restrict__ kc,
+                             const float* __restrict__ vc, RowOut att, int n, int start,
+                             int d, int kvd, int H, int Hkv, float scale, int tiles_per_split,
+                             float* __restrict__ part) {
+  constexpr int hd = 4 * kDpt, hp = hd + 4, hd4 = kDpt, nv = kDpt / 8;
+  static_assert(kDpt % 8 == 0, "head_dim must be a multiple of 32");
+  extern __shared__ __align__(16) float sm[];
+  float* Qs = sm;                       // [64][hp], q * scale
+  float* Ks = Qs + kAtt2BQ * hp;        // [32][hp]
+  float* Vs = Ks + kAttBK * hp;         // [32][hp]
+  float* Ps = Vs + kAttBK * hp;         // [64][33] softmax weights of the tile
+  const int h = blockIdx.y, kvh = h / (H / Hkv);
+  const int i0 = blockIdx.x * kAtt2BQ;
+  const int tid = threadIdx.x, g = tid >> 3, j = tid & 7;
+  const size_t rowlen = (size_t)d + 2 * kvd;
+  const int last = min(start + i0 + kAtt2BQ - 1, start + n - 1);  // the block's last position
+  const int k_begin = blockIdx.z * tiles_per_split * kAttBK;
+  if (k_begin > last) return;  // this split holds no key of these rows (uniform in the CTA)
+  const int k_end = min(last, k_begin + tiles_per_split * kAttBK - 1);
+  for (int e = tid; e < kAtt2BQ * hd4; e += kAttThreads) {
+    const int r = e / hd4, c = e - r * hd4;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (i0 + r < n) v = reinterpret_cast<const float4*>(qkv + (size_t)(i0 + r) * rowlen + h * hd)[c];
+    reinterpret_cast<float4*>(Qs + r * hp)[c] =
+        make_float4(v.x * scale, v.y * scale, v.z * scale, v.w * scale);
+  }
+  float m[4], l[4];
+  float4 o[4][nv];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    m[i] = -INFINITY;
+    l[i] = 0.f;
+#pragma unroll
+    for (int u = 0; u < nv; ++u) o[i][u] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  for (int t0 = k_begin; t0 <= k_end; t0 += kAttBK) {
+    __syncthreads();  // the previous tile's K and V are read (and Q written, the first time)
+    for (int e = tid; e < kAttBK * hd4; e += kAttThreads) {
+      const int r = e / hd4, c = e - r * hd4, t = t0 + r;
+      float4 kv = make_float4(0.f, 0.f, 0.f, 0.f), vv = kv;
+      if (t <= k_end) {
+        kv = reinterpret_cast<const float4*>(kc + (size_t)t * kvd + kvh * hd)[c];
+        vv = reinterpret_cast<const float4*>(vc + (size_t)t * kvd + kvh * hd)[c];
+      }
+      reinterpret_cast<float4*>(Ks + r * hp)[c] = kv;
+      reinterpret_cast<float4*>(Vs + r * hp)[c] = vv;
+    }
+    __syncthreads();
+    float s[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) s[i][jj] = 0.f;
+#pragma unroll 2
+    for (int c = 0; c < hd4; ++c) {
+      float4 qv[4], kv[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) qv[i] = reinterpret_cast<const float4*>(Qs + (4 * g + i) * hp)[c];
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) kv[jj] = reinterpret_cast<const float4*>(Ks + (j + 8 * jj) * hp)[c];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj)
+          s[i][jj] = fmaf(qv[i].x, kv[jj].x, fmaf(qv[i].y, kv[jj].y,
+                     fmaf(qv[i].z, kv[jj].z, fmaf(qv[i].w, kv[jj].w, s[i][jj]))));
+    }
+    // online softmax per query over the eight lanes of the group
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int qpos = start + i0 + 4 * g + i;
+      float mt = -INFINITY;
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) {
+        if (t0 + j + 8 * jj > qpos) s[i][jj] = -INFINITY;  // causal: keys after the query
+        mt = fmaxf(mt, s[i][jj]);
+      }
+      mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 1));
+      mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 2));
+      mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 4));
+      // a query whose keys so far in this split are all after it has no
+      // maximum yet (mn = -inf): nothing to add and nothing to rescale
+      const float mn = fmaxf(m[i], mt);
+      const bool none = mn == -INFINITY;
+      const float corr = none ? 1.f : expf(m[i] - mn);
+      float ps = 0.f;
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) {
+        const float e = none ? 0.f : expf(s[i][jj] - mn);
+        Ps[(4 * g + i) * (kAttBK + 1) + j + 8 * jj] = e;
+        ps += e;
+      }
+      ps += __shfl_xor_sync(0xffffffffu, ps, 1);
+      ps += __shfl_xor_sync(0xffffffffu, ps, 2);
+      ps += __shfl_xor_sync(0xffffffffu, ps, 4);
+      l[i] = l[i] * corr + ps;
+      m[i] = mn;
+#pragma unroll
+      for (int u = 0; u < nv; ++u) {
+        o[i][u].x *= corr;
+        o[i][u].y *= corr;
+        o[i][u].z *= corr;
+        o[i][u].w *= corr;
+      }
+    }
+    __syncwarp();  // the group's weights are written by lanes of this warp
+#pragma unroll 2
+    for (int k = 0; k < kAttBK; ++k) {
+      float p[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) p[i] = Ps[(4 * g + i) * (kAttBK + 1) + k];
+      const float4* vr = reinterpret_cast<const float4*>(Vs + k * hp);
+#pragma unroll
+      for (int u = 0; u < nv; ++u) {
+        const float4 v = vr[j + 8 * u];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          o[i][u].x = fmaf(p[i], v.x, o[i][u].x);
+          o[i][u].y = fmaf(p[i], v.y, o[i][u].y);
+          o[i][u].z = fmaf(p[i], v.z, o[i][u].z);
+          o[i][u].w = fmaf(p[i], v.w, o[i][u].w);
+        }
+      }
+    }
+    __syncwarp();  // the weights are read before the next tile writes them
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int row = i0 + 4 * g + i;
+    if (row >= n) continue;
+    if (part) {  // partial of split z: o (unnormalised), then max and sum
+      float* pr = part + (((size_t)blockIdx.z * n + row) * H + h) * (hd + 4);
+#pragma unroll
+      for (int u = 0; u < nv; ++u) reinterpret_cast<float4*>(pr)[j + 8 * u] = o[i][u];
+      if (j == 0) {
+        pr[hd] = m[i];
+        pr[hd + 1] = l[i];
+      }
+    } else {
+      const float inv = 1.0f / l[i];
+      const size_t out = (size_t)row * d + h * hd;
+#pragma unroll
+      for (int u = 0; u < nv; ++u) {
+        const size_t e = out + 4 * (j + 8 * u);
+        att.put(e, o[i][u].x * inv);
+        att.put(e + 1, o[i][u].y * inv);
+        att.put(e + 2, o[i][u].z * inv);
+        att.put(e + 3, o[i][u].w * inv);
+      }
+    }
+  }
+}
+
 // Combines the key splits of attention_tiles_kernel, one warp per (row, head):
 // o = sum_z e^(m_z - M) o_z / sum_z e^(m_z - M) l_z, M = max_z m_z, over the
 // splits that hold keys of the row's 32-row block (split 0 holds key 0 of every
@@ -376,6 +545,32 @@ tvl_status launch_attention_tiles(const float* qkv, const float* kc, const float
   const int nsplit = (ntiles + tps - 1) / tps;
   const dim3 grid((n + kAttBQ - 1) / kAttBQ, H, nsplit);
   attention_tiles_kernel<kDpt><<<grid, kAttThreads, smem, st>>>(
+      qkv, kc, vc, att, n, start, d, kvd, H, Hkv, scale, tps, nsplit > 1 ? part : nullptr);
+  TVL_CK(cudaGetLastError());
+  if (nsplit > 1) {
+    const int warps = n * H, wpb = kRowThreads / 32;
+    attention_merge_kernel<<<(warps + wpb - 1) / wpb, kRowThreads, 0, st>>>(part, att, n, start, d,
+                                                                           H, 4 * kDpt, tps);
+    TVL_CK(cudaGetLastError());
+  }
+  return TVL_OK;
+}
+
+template <int kDpt>
+tvl_status launch_attention_tiles64(const float* qkv, const float* kc, const float* vc,
+                                    RowOut att, int n, int start, int d, int kvd, int H, int Hkv,
+                                    float scale, float* part, cudaStream_t st) {
+  constexpr int hp = 4 * kDpt + 4;
+  const int smem =
+      (int)(sizeof(float) * ((kAtt2BQ + 2 * kAttBK) * hp + kAtt2BQ * (kAttBK + 1)));
+  TVL_CK(cudaFuncSetAttribute((const void*)attention_tiles64_kernel<kDpt>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+  const int ntiles = (start + n + kAttBK - 1) / kAttBK;
+  int tps = (ntiles + kAttSplits - 1) / kAttSplits;
+  if (tps < 4) tps = 4;
+  const int nsplit = (ntiles + tps - 1) / tps;
+  const dim3 grid((n + kAtt2BQ - 1) / kAtt2BQ, H, nsplit);
+  attention_tiles64_kernel<kDpt><<<grid, kAttThreads, smem, st>>>(
       qkv, kc, vc, att, n, start, d, kvd, H, Hkv, scale, tps, nsplit > 1 ? part : nullptr);
   TVL_CK(cudaGetLastError());
   if (nsplit > 1) {
@@ -528,18 +723,19 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
       return s;
     rope_kv_kernel<<<n, kRowThreads, 0, st>>>(QKV, a.rope, kc, vc, start_pos, d, kvd, hd);
     TVL_CK(cudaGetLastError());
-    {  // head dims of 16 to 128 in steps of 16 take the tiled kernel
+    {  // head dims of 16 to 128 in steps of 16 take a tiled kernel (multiples of 32:
+       // 64 queries per CTA, register blocks; the others: 32 queries per CTA)
       const float sc = a.att_scale;
       s = TVL_OK;
       switch (hd) {
         case 16: s = launch_attention_tiles<4>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
-        case 32: s = launch_attention_tiles<8>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 32: s = launch_attention_tiles64<8>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
         case 48: s = launch_attention_tiles<12>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
-        case 64: s = launch_attention_tiles<16>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 64: s = launch_attention_tiles64<16>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
         case 80: s = launch_attention_tiles<20>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
-        case 96: s = launch_attention_tiles<24>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 96: s = launch_attention_tiles64<24>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
         case 112: s = launch_attention_tiles<28>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
-        case 128: s = launch_attention_tiles<32>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
+        case 128: s = launch_attention_tiles64<32>(QKV, kc, vc, parts, n, start_pos, d, kvd, a.H, a.Hkv, sc, PART, st); break;
         default: {
           const int warps = n * a.H, wpb = kRowThreads / 32;
           attention_rows_kernel<<<(warps + wpb - 1) / wpb, kRowThreads, 0, st>>>(

@@ -57,7 +57,9 @@ def check_prefill_then_decode(tvl, cfg, blob, n, n_decode=8, label=""):
     dict(n_layers=0),                          # embedding -> final norm -> classifier
     dict(dim=96, n_heads=2, n_kv_heads=2, hidden_dim=8200, vocab_size=333),  # wide FFN
     dict(dim=128, n_heads=1, n_kv_heads=1, hidden_dim=256),  # head_dim 128
-], ids=["base", "gqa2", "mqa", "L0", "wide_ffn", "hd128"])
+    dict(n_heads=2, n_kv_heads=1),                           # head_dim 32, grouped
+    dict(dim=192, n_heads=2, n_kv_heads=2, hidden_dim=128),  # head_dim 96
+], ids=["base", "gqa2", "mqa", "L0", "wide_ffn", "hd128", "hd32_gqa", "hd96"])
 def test_prefill_matches_oracle(tvl, kw):
     cfg = small_config(**kw)
     blob = synth.make_blob(cfg, seed=41)
@@ -132,7 +134,8 @@ def test_110m_prefill_896_prompt_then_greedy(tvl):
     ((300, 140), dict()),                                     # 14 key tiles: 4 splits of 4
     ((1050,), dict(dim=128, n_heads=2, n_kv_heads=1)),        # 33 tiles: 7 splits of 5, hd 64
     ((129, 3, 700), dict(n_kv_heads=2)),                      # ragged parts, grouped heads
-], ids=["two_parts", "long_hd64", "ragged"])
+    ((65, 1, 300, 130), dict(dim=128, n_heads=2, n_kv_heads=1)),  # ragged, head_dim 64
+], ids=["two_parts", "long_hd64", "ragged", "ragged_hd64"])
 def test_prefill_long_key_ranges_split_across_ctas(tvl, parts, kw):
     """Rows that see more than 128 keys have their key range cut into up to
     eight parts, each a CTA of its own, whose partial sums are merged; the
