@@ -508,24 +508,25 @@ __global__ void attention_merge_kernel(const float* __restrict__ part, RowOut at
   if (gw >= n * H) return;
   const int lane = threadIdx.x & 31, i = gw / H, h = gw - i * H;
   const int last = min(start + (i / kAttBQ) * kAttBQ + kAttBQ - 1, start + n - 1);
-  const int nz = last / (tiles_per_split * kAttBK) + 1;
+  const int nz = last / (tiles_per_split * kAttBK) + 1;  // at most kAttSplits
   const size_t stride = (size_t)n * H * (hd + 4);
   const float* p0 = part + ((size_t)i * H + h) * (hd + 4);
-  float M = -INFINITY;
-  for (int z = 0; z < nz; ++z) M = fmaxf(M, p0[z * stride + hd]);
-  float L = 0.f;
-  for (int z = 0; z < nz; ++z) {
-    const float mz = p0[z * stride + hd];
-    if (mz != -INFINITY) L += expf(mz - M) * p0[z * stride + hd + 1];
-  }
-  const float inv = 1.0f / L;
-  for (int j = lane; j < hd; j += 32) {
+  // lane z < nz holds split z's max and sum; every load below is issued at once
+  const float mz = lane < nz ? p0[lane * stride + hd] : -INFINITY;
+  const float lz = lane < nz ? p0[lane * stride + hd + 1] : 0.f;
+  float M = mz;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  const float wz = mz == -INFINITY ? 0.f : expf(mz - M);
+  const float inv = 1.0f / warp_sum32(wz * lz);
+  for (int jj = lane; jj < hd; jj += 32) {
+    float v[kAttSplits];
+#pragma unroll
+    for (int z = 0; z < kAttSplits; ++z) v[z] = z < nz ? p0[z * stride + jj] : 0.f;
     float o = 0.f;
-    for (int z = 0; z < nz; ++z) {
-      const float mz = p0[z * stride + hd];
-      if (mz != -INFINITY) o = fmaf(expf(mz - M), p0[z * stride + j], o);
-    }
-    att.put((size_t)i * d + h * hd + j, o * inv);
+#pragma unroll
+    for (int z = 0; z < kAttSplits; ++z) o = fmaf(__shfl_sync(0xffffffffu, wz, z), v[z], o);
+    att.put((size_t)i * d + h * hd + jj, o * inv);
   }
 }
 
