@@ -121,3 +121,23 @@ def test_reference_arm_config_equals_the_gpu_arms(capsys):
     wins = bench.timed_windows(64, 3, 0)
     assert line["config"] == bench.workload_config("tiny", cfg, 1, "f32", bench.positions_of(wins))
     assert line["config"]["positions"] == [[30, 32]]
+
+
+def test_streamed_bytes_per_step_by_weight_format():
+    # The weights one decode step reads, worked out by hand for the 110M shape
+    # (d 768, L 12, F 2048, V 32000, tied): float32 rows 4 bytes a value;
+    # quantized rows 16 bytes of scale and padding plus the codes (K bytes for
+    # 8-bit, K / 2 for 4-bit); the gains, one embedding row and the final gain
+    # stay float32 (4-bit: (2304 + 768 + 4096) * 400 + 768 * 1040 + 8 * 768 =
+    # 3,672,064 bytes per layer; 12 layers, then 32000 classifier rows of 400
+    # bytes, one embedding row of 400 and the final gain's 3072).
+    import bench
+    from paper_2601_03324_gb300 import synth
+    cfg = synth.model_config("110m")
+    assert bench.streamed_bytes_of(cfg, 0) == 4 * (12 * (2304 * 768 + 768 * 768 + 3 * 2048 * 768
+                                                        + 2 * 768) + 32000 * 768 + 2 * 768)
+    assert bench.streamed_bytes_of(cfg, 0) == 438_122_496
+    assert bench.streamed_bytes_of(cfg, 8) == 12 * ((2304 + 768 + 4096) * 784 + 768 * 2064
+                                                    + 8 * 768) + 32000 * 784 + 784 + 3072
+    assert bench.streamed_bytes_of(cfg, 4) == 12 * 3_672_064 + 32000 * 400 + 400 + 3072
+    assert bench.streamed_bytes_of(cfg, 4) == 56_868_240
