@@ -143,6 +143,19 @@ bool is_device_pointer(const void* p) {
   return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
 }
 
+// The device address of pinned, mapped host memory (cudaHostAlloc, or
+// registered with cudaHostRegister), else null: the kernel can store there
+// directly, with no copy after it.
+float* mapped_host_pointer(void* p) {
+  cudaPointerAttributes at{};
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  if (at.type != cudaMemoryTypeHost || !at.devicePointer) return nullptr;
+  return static_cast<float*>(at.devicePointer);
+}
+
 // Interleaves the rows of a [W1 | W3] block in place (F rows of row_bytes
 // each, then F more): row 2i becomes W1's row i and row 2i + 1 W3's, so that
 // one CTA computes both halves of each SwiGLU product. tmp holds the block.
@@ -158,8 +171,9 @@ tvl_status interleave_w13(unsigned char* block, size_t F, size_t row_bytes, unsi
 }
 
 tvl_status launch(tvl_model* m, int B, const int* tokens, int pos, int n_steps,
-                  int final_token) {
+                  int final_token, float* logits_dst = nullptr) {
   DecodeArgs a = m->args;
+  if (logits_dst) a.logits = logits_dst;  // the classifier writes there directly
   for (int b = 0; b < B; ++b) a.start_tokens[b] = tokens[b];
   a.start_pos = pos;
   a.n_steps = n_steps;
@@ -586,9 +600,15 @@ tvl_status tvl_forward_batch(tvl_model* m, int32_t batch, const int32_t* tokens,
     set_error("tvl_forward_batch: position out of range");
     return TVL_E_RANGE;
   }
-  tvl_status st = launch(m, batch, tokens, pos, 1, 0);
+  // pinned host logits: the classifier's epilogue writes them in place
+  float* mapped = logits_out ? mapped_host_pointer(logits_out) : nullptr;
+  tvl_status st = launch(m, batch, tokens, pos, 1, 0, mapped);
   if (st != TVL_OK) return st;
   if (!logits_out) return TVL_OK;
+  if (mapped) {
+    TVL_CK(cudaStreamSynchronize(m->stream));
+    return check_device_error(m);
+  }
   const size_t bytes = (size_t)m->cfg.vocab_size * 4 * batch;
   if (is_device_pointer(logits_out)) {
     TVL_CK(cudaMemcpyAsync(logits_out, m->args.logits, bytes, cudaMemcpyDeviceToDevice,

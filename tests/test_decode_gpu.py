@@ -94,6 +94,31 @@ def test_device_logits_pointer_and_repeat_are_bitwise_stable(tvl):
         assert np.array_equal(dl.cpu().numpy(), h1)
 
 
+def test_pinned_host_logits_are_written_by_the_kernel_itself(tvl):
+    # A pinned (mapped) host buffer receives the logits from the classifier
+    # phase directly, with no copy after the kernel: the same bits as the
+    # device copy, oracle parity along a teacher-forced run, and the batched
+    # form laid out [batch][V].
+    cfg = small_config(max_batch=2)
+    blob = synth.make_blob(cfg, seed=6)
+    V = cfg["vocab_size"]
+    ref = oracle.Model(cfg, blob, 64)
+    pinned = torch.empty(2 * V, dtype=torch.float32, pin_memory=True).numpy()
+    pageable = np.empty(2 * V, np.float32)
+    with tvl.Model(cfg, blob) as m:
+        t = 1
+        for p in range(12):
+            m.forward(t, p, pinned)
+            lg = ref.forward(t, p)
+            assert_logits_close(pinned[:V], lg, f"pinned pos {p}")
+            m.forward(t, p, pageable)  # the same position again: the same bits
+            assert np.array_equal(pinned[:V], pageable[:V])
+            t = int(np.argmax(lg))
+        m.forward_batch([5, 7], 0, pinned)
+        m.forward_batch([5, 7], 0, pageable)
+        assert np.array_equal(pinned, pageable)
+
+
 def test_out_of_range_arguments(tvl):
     cfg = small_config(max_seq=8)
     blob = synth.make_blob(cfg, seed=2)
