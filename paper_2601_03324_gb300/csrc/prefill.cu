@@ -34,6 +34,24 @@ struct RowOut {
     if (hi) store_bf16_parts(hi, lo, i, v);
     else f[i] = v;
   }
+  // four values at i, a multiple of 4: one 16-byte or two 8-byte stores
+  __device__ __forceinline__ void put4(size_t i, float4 v) const {
+    if (hi) {
+      const __nv_bfloat162 h01 = __floats2bfloat162_rn(v.x, v.y), h23 = __floats2bfloat162_rn(v.z, v.w);
+      const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+      const __nv_bfloat162 l01 = __floats2bfloat162_rn(v.x - f01.x, v.y - f01.y);
+      const __nv_bfloat162 l23 = __floats2bfloat162_rn(v.z - f23.x, v.w - f23.y);
+      uint2 hv, lv;
+      hv.x = *reinterpret_cast<const unsigned*>(&h01);
+      hv.y = *reinterpret_cast<const unsigned*>(&h23);
+      lv.x = *reinterpret_cast<const unsigned*>(&l01);
+      lv.y = *reinterpret_cast<const unsigned*>(&l23);
+      *reinterpret_cast<uint2*>(hi + i) = hv;
+      *reinterpret_cast<uint2*>(lo + i) = lv;
+    } else {
+      *reinterpret_cast<float4*>(f + i) = v;
+    }
+  }
 };
 
 __device__ __forceinline__ float warp_sum32(float v) {
@@ -60,15 +78,19 @@ __global__ void rmsnorm_rows_kernel(float* x, const float* add, const float* __r
                                     RowOut out, int row0, int d, float eps) {
   __shared__ float red[kRowThreads / 32];
   const int i = row0 + blockIdx.x;
-  float* xr = x + (size_t)i * d;
+  float4* xr = reinterpret_cast<float4*>(x + (size_t)i * d);  // d % 32 == 0
+  const float4* ar = add ? reinterpret_cast<const float4*>(add + (size_t)i * d) : nullptr;
+  const float4* g4 = reinterpret_cast<const float4*>(g);
+  const int d4 = d >> 2;
   float ss = 0.f;
-  for (int j = threadIdx.x; j < d; j += blockDim.x) {
-    float v = xr[j];
-    if (add) {
-      v += add[(size_t)i * d + j];
+  for (int j = threadIdx.x; j < d4; j += blockDim.x) {
+    float4 v = xr[j];
+    if (ar) {
+      const float4 u = ar[j];
+      v = make_float4(v.x + u.x, v.y + u.y, v.z + u.z, v.w + u.w);
       xr[j] = v;
     }
-    ss = fmaf(v, v, ss);
+    ss = fmaf(v.x, v.x, fmaf(v.y, v.y, fmaf(v.z, v.z, fmaf(v.w, v.w, ss))));
   }
   ss = warp_sum32(ss);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
@@ -77,7 +99,14 @@ __global__ void rmsnorm_rows_kernel(float* x, const float* add, const float* __r
   for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += red[w];
   const float r = 1.0f / sqrtf(tot / (float)d + eps);
   const size_t o = (size_t)blockIdx.x * d;
-  for (int j = threadIdx.x; j < d; j += blockDim.x) out.put(o + j, (g ? xr[j] * g[j] : xr[j]) * r);
+  for (int j = threadIdx.x; j < d4; j += blockDim.x) {
+    float4 v = xr[j];
+    if (g4) {
+      const float4 gg = g4[j];
+      v = make_float4(v.x * gg.x, v.y * gg.y, v.z * gg.z, v.w * gg.w);
+    }
+    out.put4(o + 4 * j, make_float4(v.x * r, v.y * r, v.z * r, v.w * r));
+  }
 }
 
 // RoPE on q and k of row i (position start + i): pair (2m, 2m+1) of a head
@@ -586,11 +615,18 @@ tvl_status launch_attention_tiles64(const float* qkv, const float* kc, const flo
 // h[i][j] = silu(a) * b with (a, b) = rows (2j, 2j + 1) of the interleaved
 // W1/W3 output (§2.1, SwiGLU).
 __global__ void swiglu_rows_kernel(const float* __restrict__ h13, RowOut h, long long total) {
-  for (long long t = blockIdx.x * (long long)blockDim.x + threadIdx.x; t < total;
+  auto silu_mul = [](float a, float b) { return (a / (1.0f + expf(-a))) * b; };
+  const long long t4 = total >> 2;  // four outputs from eight inputs at a time
+  const float4* in = reinterpret_cast<const float4*>(h13);
+  for (long long t = blockIdx.x * (long long)blockDim.x + threadIdx.x; t < t4;
        t += (long long)gridDim.x * blockDim.x) {
-    const float a = h13[2 * t], b = h13[2 * t + 1];
-    h.put((size_t)t, (a / (1.0f + expf(-a))) * b);
+    const float4 p = in[2 * t], q = in[2 * t + 1];
+    h.put4((size_t)(4 * t), make_float4(silu_mul(p.x, p.y), silu_mul(p.z, p.w),
+                                         silu_mul(q.x, q.y), silu_mul(q.z, q.w)));
   }
+  for (long long t = 4 * t4 + blockIdx.x * (long long)blockDim.x + threadIdx.x; t < total;
+       t += (long long)gridDim.x * blockDim.x)
+    h.put((size_t)t, silu_mul(h13[2 * t], h13[2 * t + 1]));
 }
 
 // The bf16 parts (hi then lo) of one weight matrix [M x K] in the prefill's
@@ -752,8 +788,8 @@ extern "C" tvl_status tvl_prefill(tvl_model* m, const int32_t* tokens, int32_t n
     TVL_CK(cudaGetLastError());
     if ((s = gemm_rows(wparts(l, 2), xh, xl, H13, n, 2 * F, d, err, st)) != TVL_OK) return s;
     const long long tot = (long long)n * F;
-    swiglu_rows_kernel<<<(int)std::min<long long>((tot + 255) / 256, 4096), 256, 0, st>>>(H13, parts,
-                                                                                        tot);
+    swiglu_rows_kernel<<<(int)std::min<long long>((tot / 4 + 255) / 256 + 1, 4096), 256, 0, st>>>(
+        H13, parts, tot);
     TVL_CK(cudaGetLastError());
     // Y = W2 h
     if ((s = gemm_rows(wparts(l, 3), xh, xl, Y, n, d, F, err, st)) != TVL_OK) return s;
