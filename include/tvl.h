@@ -103,9 +103,10 @@ tvl_status tvl_load_file(const tvl_config* cfg, const char* path, void* stream, 
  *   calling a position again overwrites it).
  *   logits_out: V floats. Device pointer: the copy is queued on the model
  *   stream and the call returns without waiting. Host pointer: the call waits
- *   and then reports device-side errors; pinned, mapped host memory
- *   (cudaHostAlloc, cudaHostRegister) is written by the kernel itself, other
- *   host memory by a copy after it. NULL: logits stay on the device.
+ *   and then reports device-side errors; pinned, mapped, writable host
+ *   memory (cudaHostAlloc, cudaHostRegister without the read-only flag) is
+ *   written by the kernel itself, other host memory by a copy after it.
+ *   NULL: logits stay on the device.
  * The whole step is one kernel launch (a persistent kernel). */
 tvl_status tvl_forward(tvl_model* m, int32_t token, int32_t pos, float* logits_out);
 
